@@ -1,0 +1,411 @@
+"""Benchmark of the VarRate hot path on GB300.
+
+One step = one pass of the whole hot path over one batch of synthetic input:
+  encode (salience -> rank allocation -> projection/packing) of every (sequence, layer), then
+  ``decode_steps`` decode steps, each running decode attention on the packed coefficients of every
+  layer for every sequence.
+
+Default workload (N=1): the Llama-3.1-8B-shaped full KV stack — 32 layers x 8 KV heads, 32 query
+heads, head_dim 128, N = 32768, bf16, budget 0.20, r_min 16, window 32, 8 independent sequences,
+256 decode steps. Its packed cache (~6.9 GB read per decode step) is far larger than L2, so no L2
+flush is needed between timed iterations.
+
+Reported: ``value`` = decode-attention GB/s (algorithmic bytes: the stored coefficients sum_t r_t
+of K and V in bf16, plus the per-head bases, queries and outputs) over the timed decode phase of
+all steps, with inputs resident in HBM; ``encode_ms_per_32k_ctx`` = encode time per sequence
+(32 layers x 32768 tokens). ``e2e`` repeats the measurement through the same C ABI with the inputs
+in pinned host memory and host<->device copies inside the timed region.
+
+``--impl reference`` times the CPU oracle (the only reference this method has) on a bounded
+sample of the same workload and prints the same JSON line with ``"impl": "reference"``.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+METRIC = "decode-attn GB/s (% of HBM peak) over packed cache; encode ms per 32k ctx"
+FALLBACK_HBM_GBS = 6800.0
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    return FALLBACK_HBM_GBS, "fallback"
+
+
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+class Clocks:
+    """nvidia-smi sampled every 200 ms during the timed region."""
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.QUERY}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i] == "Active"})
+        power = [float(r[3]) for r in rows if r[3].replace(".", "").isdigit()]
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons,
+                "samples": len(rows), "power_w_max": max(power) if power else None}
+
+
+# ------------------------------------------------------------------------ our CUDA path
+
+def algorithmic_decode_bytes(packed, cfg, elem=2):
+    """Bytes one decode call (one layer, all sequences) must move: K and V coefficients
+    (sum of ranks, no padding) of every head, the two bases, queries and outputs."""
+    d = cfg.head_dim
+    cnt = packed.bucket_count.to(torch.int64).cpu()                   # [B][L][d+1]
+    ranks_sum = (cnt * torch.arange(d + 1)).sum(-1)                      # [B][L]
+    per_layer = ranks_sum.sum(0) * cfg.n_kv_heads * 2 * elem            # [L]
+    basis = 2 * cfg.n_kv_heads * d * d * elem
+    qo = 2 * cfg.batch * cfg.n_kv_heads * cfg.group * d * elem
+    return (per_layer + basis + qo).tolist()
+
+
+def run_ours(args, wl, rank, world):
+    from paper_2607_15498_gb300 import varrate as V
+    V.lib()
+    dev = torch.device("cuda", torch.cuda.current_device())
+    cfg = V.make_config(wl.n_layers, wl.n_kv_heads, wl.group, wl.n_ctx, batch=wl.batch,
+                        budget_frac=wl.budget_frac, r_min=wl.r_min, window=wl.window,
+                        dtype=V.BF16 if wl.dtype == "bf16" else V.F32)
+    D = args.decode_steps
+    L, B = wl.n_layers, wl.batch
+    # inputs drawn on the device (seeded; rank r draws sequences of batch index r)
+    k, v, qw, bk, bv = synth.stack_inputs(wl, device=dev, batch_index=rank)
+    qdec = torch.stack([synth.stack_decode_queries(wl, l, D, device=dev, batch_index=rank)
+                        for l in range(L)], dim=1)                       # [D][L][B][H][d]
+    packed = V.PackedCache.allocate(cfg, dev)
+    realized = torch.zeros((B, L), dtype=torch.int64, device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    ws_enc = V.workspace(cfg, V.CALL_ENCODE, dev)
+    ws_dec = V.workspace(cfg, V.CALL_DECODE, dev)
+    out = torch.empty((B, wl.n_q_heads, wl.head_dim), dtype=k.dtype, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def encode():
+        V.check(V.varrate_encode(cfg, qw, k, v, bk, bv, None, packed, realized, status, ws_enc,
+                                 stream), "varrate_encode")
+
+    def decode_phase(evs=None):
+        i = 0
+        for s in range(D):
+            for l in range(L):
+                if evs is not None:
+                    evs[i].record(stream)
+                    i += 1
+                V.check(V.varrate_decode_attn(cfg, packed, bk, bv, qdec[s, l], l, None, None, 0,
+                                              out, status, ws_dec, stream), "varrate_decode_attn")
+        if evs is not None:
+            evs[i].record(stream)
+
+    for _ in range(args.warmup):
+        encode()
+        decode_phase()
+    torch.cuda.synchronize()
+    st = int(status.item())
+    if st < 0:
+        raise RuntimeError(f"device status {st}: {V.status_string(st)}")
+    dec_bytes = algorithmic_decode_bytes(packed, cfg)                  # per layer call
+    step_dec_bytes = D * sum(dec_bytes)
+
+    n_calls = D * L
+    call_evs = [torch.cuda.Event(enable_timing=True) for _ in range(n_calls + 1)]
+    e_beg = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    e_mid = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    call_ms = []
+    clocks = Clocks(torch.cuda.current_device())
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for i in range(args.steps):
+        e_beg[i].record(stream)
+        encode()
+        e_mid[i].record(stream)
+        decode_phase(call_evs)
+        # per-call durations of this step (host waits only for the events of this step)
+        call_evs[-1].synchronize()
+        call_ms.append([call_evs[j].elapsed_time(call_evs[j + 1]) for j in range(n_calls)])
+    t1.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    clk = clocks.stop()
+    total_ms = t0.elapsed_time(t1)
+    enc_ms = [e_beg[i].elapsed_time(e_mid[i]) for i in range(args.steps)]
+    dec_ms = [sum(c) for c in call_ms]
+
+    # e2e: same calls, inputs in pinned host memory, copies inside the timed region
+    e2e = None
+    if not args.no_e2e:
+        e2e = run_e2e(args, V, cfg, wl, k, v, qw, bk, bv, qdec, packed, realized, status, ws_enc,
+                      ws_dec, stream, dec_bytes)
+    st = int(status.item())
+    if st < 0:
+        raise RuntimeError(f"device status {st}: {V.status_string(st)}")
+    return dict(total_ms=total_ms, enc_ms=enc_ms, dec_ms=dec_ms, call_ms=call_ms,
+                step_dec_bytes=step_dec_bytes, dec_bytes=dec_bytes, clocks=clk, e2e=e2e,
+                launches_per_step=6 + 3 * n_calls, realized=realized.cpu(), status=st)
+
+
+def run_e2e(args, V, cfg, wl, k, v, qw, bk, bv, qdec, packed, realized, status, ws_enc, ws_dec,
+            stream, dec_bytes):
+    D, L = args.decode_steps, wl.n_layers
+    steps = max(1, min(args.steps, args.e2e_steps))
+    hk = torch.empty(k.shape, dtype=k.dtype, pin_memory=True)
+    hv = torch.empty(v.shape, dtype=v.dtype, pin_memory=True)
+    hq = torch.empty(qw.shape, dtype=qw.dtype, pin_memory=True)
+    hqd = torch.empty(qdec.shape, dtype=qdec.dtype, pin_memory=True)
+    hk.copy_(k)
+    hv.copy_(v)
+    hq.copy_(qw)
+    hqd.copy_(qdec)
+    dk, dv, dq = torch.empty_like(k), torch.empty_like(v), torch.empty_like(qw)
+    dqs = torch.empty_like(qdec[0, 0])
+    dout = torch.empty((cfg.batch, wl.n_q_heads, wl.head_dim), dtype=k.dtype, device=k.device)
+    hout = torch.empty(dout.shape, dtype=dout.dtype, pin_memory=True)
+    torch.cuda.synchronize()
+
+    def one_step(evs):
+        evs[0].record(stream)
+        dk.copy_(hk, non_blocking=True)
+        dv.copy_(hv, non_blocking=True)
+        dq.copy_(hq, non_blocking=True)
+        V.check(V.varrate_encode(cfg, dq, dk, dv, bk, bv, None, packed, realized, status, ws_enc,
+                                 stream))
+        evs[1].record(stream)
+        for s in range(D):
+            for l in range(L):
+                dqs.copy_(hqd[s, l], non_blocking=True)
+                V.check(V.varrate_decode_attn(cfg, packed, bk, bv, dqs, l, None, None, 0, dout,
+                                              status, ws_dec, stream))
+                hout.copy_(dout, non_blocking=True)
+        evs[2].record(stream)
+
+    one_step([torch.cuda.Event(enable_timing=True) for _ in range(3)])   # warm
+    torch.cuda.synchronize()
+    enc, dec = [], []
+    for _ in range(steps):
+        evs = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+        one_step(evs)
+        torch.cuda.synchronize()
+        enc.append(evs[0].elapsed_time(evs[1]))
+        dec.append(evs[1].elapsed_time(evs[2]))
+    h2d = (hk.numel() + hv.numel() + hq.numel() + hqd.numel()) * hk.element_size()
+    d2h = D * L * hout.numel() * hout.element_size()
+    dec_gbs = D * sum(dec_bytes) / (statistics.mean(dec) * 1e-3) / 1e9
+    return {"value": round(dec_gbs, 1), "unit": "GB/s",
+            "encode_ms_per_32k_ctx": round(statistics.mean(enc) / cfg.batch, 3),
+            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": steps}
+
+
+# -------------------------------------------------------------------- the CPU oracle
+
+def run_oracle_sample(wl, budget_s: float = 15.0, decode_steps: int = 2, seed_layer: int = 0):
+    """Times the oracle as it stands on a bounded sample of the workload: encode of one
+    (sequence, layer) and a few decode steps of that layer. Returns rates in the bench's units."""
+    import oracle as O
+    t0 = time.perf_counter()
+    k, v = synth.layer_kv(wl, 0, seed_layer)
+    qw = synth.window_queries(wl, 0, seed_layer)
+    uk, uv = synth.basis_tensors(wl, seed_layer)
+    f64 = lambda t: t.to(torch.float64).numpy()  # noqa: E731
+    k, v, qw, uk, uv = f64(k), f64(v), f64(qw), f64(uk), f64(uv)
+    t_in = time.perf_counter() - t0
+    t0 = time.perf_counter()
+    enc = O.encode_layer(qw, k, v, uk, uv, wl.group, wl.budget_frac, wl.r_min)
+    t_enc = time.perf_counter() - t0
+    qs = synth.decode_queries(wl, 0, seed_layer, decode_steps)
+    t0 = time.perf_counter()
+    n = 0
+    for s in range(decode_steps):
+        O.decode_coef(f64(qs[s]), enc["coef_k"], enc["coef_v"], enc["ranks"], uk, uv)
+        n += 1
+        if time.perf_counter() - t0 > budget_s:
+            break
+    t_dec = (time.perf_counter() - t0) / n
+    d = wl.head_dim
+    bytes_per = int(enc["ranks"].sum()) * wl.n_kv_heads * 2 * 2 + 2 * wl.n_kv_heads * d * d * 2 \
+        + 2 * wl.n_q_heads * d * 2
+    return {"decode_gbs": bytes_per / t_dec / 1e9, "decode_s_per_layer_step": t_dec,
+            "encode_s_per_layer": t_enc, "encode_ms_per_32k_ctx": t_enc * wl.n_layers * 1e3,
+            "steps": n, "input_s": t_in}
+
+
+def cpu_cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+# ----------------------------------------------------------------------------- main
+
+def workload_desc(wl):
+    return (f"{wl.name}: {wl.n_layers} layers x {wl.n_kv_heads} KV heads, {wl.n_q_heads} query "
+            f"heads (GQA {wl.group}), head_dim {wl.head_dim}, N={wl.n_ctx}, batch {wl.batch}, "
+            f"{wl.dtype}, budget {wl.budget_frac}, r_min {wl.r_min}, window {wl.window}")
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=3)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="llama32", choices=sorted(synth.WORKLOADS))
+    ap.add_argument("--decode-steps", type=int, default=None)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--e2e-steps", type=int, default=1)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    wl = synth.workload(args.workload)
+    if args.decode_steps is None:
+        args.decode_steps = wl.decode_steps
+    world, rank, local = dist_env()
+    peak, peak_kind = measured_peaks()
+    cfg_json = {"workload": workload_desc(wl), "model": "Llama-3.1-8B-shaped KV stack (shapes only, no weights)"
+                if wl.name.startswith("llama") else wl.name,
+                "global_batch": wl.batch * world, "seq_len": wl.n_ctx,
+                "decode_steps": args.decode_steps, "parallelism": f"replicas over sequences x{world}",
+                "l2": "inputs larger than L2 (packed cache of all layers re-read every decode step)"}
+    base = {"metric": METRIC, "unit": "GB/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": wl.dtype, "data": "synthetic: seeded low-rank-plus-noise K/V, Gaussian queries",
+            "config": cfg_json}
+
+    if args.impl == "reference":
+        if rank != 0:
+            return
+        t0 = time.perf_counter()
+        vals = []
+        per_step = []
+        for i in range(args.warmup + args.steps):
+            r = run_oracle_sample(wl, budget_s=5.0, decode_steps=1, seed_layer=i % wl.n_layers)
+            if i >= args.warmup:
+                vals.append(r["decode_gbs"])
+                per_step.append(r)
+        val = statistics.mean(vals)
+        cores = cpu_cores()
+        line = dict(base, impl="reference", value=val,
+                    ms_per_step=1e3 * (time.perf_counter() - t0) / (args.warmup + args.steps),
+                    encode_ms_per_32k_ctx=statistics.mean(r["encode_ms_per_32k_ctx"] for r in per_step),
+                    cpu_baseline={"value": val, "unit": "GB/s", "cores": cores, "kind": "oracle",
+                                  "sample": "per step: encode of one (sequence, layer) and one decode "
+                                            "step of that layer, numpy fp64"},
+                    e2e={"value": val, "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0})
+        line["gpu_launches"] = 0
+        print(json.dumps(line))
+        return
+
+    if world > 1:
+        torch.distributed.init_process_group("nccl")
+        torch.cuda.set_device(local)
+    else:
+        torch.cuda.set_device(0)
+    r = run_ours(args, wl, rank, world)
+    K = args.steps
+    total_s = r["total_ms"] * 1e-3
+    dec_s = sum(r["dec_ms"]) * 1e-3
+    enc_ms_per_ctx = statistics.mean(r["enc_ms"]) / wl.batch
+    if world > 1:
+        t = torch.tensor([total_s, dec_s, enc_ms_per_ctx], dtype=torch.float64, device="cuda")
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        total_s, dec_s, enc_ms_per_ctx = t.tolist()
+    dec_gbs = world * K * r["step_dec_bytes"] / dec_s / 1e9
+    calls = [c for step in r["call_ms"] for c in step]
+    avg_call_ms = statistics.mean(calls)
+    bytes_per_call = statistics.mean(r["dec_bytes"])
+    achieved = bytes_per_call / (avg_call_ms * 1e-3) / 1e9
+    line = dict(base, value=round(dec_gbs, 1), ms_per_step=round(1e3 * total_s / K, 3),
+                encode_ms_per_32k_ctx=round(enc_ms_per_ctx, 3),
+                decode_ms_per_step=round(1e3 * dec_s / K / args.decode_steps, 4),
+                decode_frac_of_hbm_peak=round(dec_gbs / world / peak, 4),
+                decode_frac_of_nominal_8tbs=round(dec_gbs / world / 8000.0, 4),
+                roofline={"bound": "hbm", "kernel": "varrate_decode_attn (rotate + split + combine)",
+                          "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+                          "frac": round(achieved / peak, 4), "traffic": None,
+                          "peak_source": f"{peak_kind} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)"
+                          if peak_kind == "measured" else "fallback 6.8 TB/s",
+                          "bytes_per_launch": int(bytes_per_call),
+                          "avg_launch_us": round(avg_call_ms * 1e3, 2)},
+                gpu_launches=int(r["launches_per_step"] * K), clocks=r["clocks"],
+                e2e=r["e2e"])
+    if rank == 0 and not args.no_cpu_baseline:
+        cb = run_oracle_sample(wl, budget_s=10.0, decode_steps=2)
+        line["cpu_baseline"] = {"value": cb["decode_gbs"], "unit": "GB/s", "cores": cpu_cores(),
+                                "kind": "oracle", "encode_ms_per_32k_ctx": cb["encode_ms_per_32k_ctx"],
+                                "sample": f"encode of 1 (sequence, layer) of {wl.n_layers * wl.batch} "
+                                          f"and {cb['steps']} decode step(s) of that layer, numpy fp64"}
+    if rank == 0:
+        print(json.dumps(line))
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,182 @@
+/*
+ * varrate.h — C ABI of the GB300 (sm_103a) VarRate hot path.
+ *
+ * VarRate (arXiv 2607.15498) compresses a KV cache by giving every cached token its own rank in
+ * a fixed orthonormal basis: salience from an observation window decides how many basis
+ * coefficients each token keeps (Sec. 3.2), the coefficients are the projection onto the basis
+ * truncated to that rank (Sec. 3.3, Eq. 5), and decode attention runs directly on the stored
+ * coefficients with the query rotated into the basis.
+ *
+ * Conventions shared by every entry point
+ *  - Every tensor argument is a caller-owned DEVICE pointer (CUDA global memory), row-major and
+ *    densely packed in the layout stated next to it. The library never allocates or frees device
+ *    memory and keeps no state between calls (reentrant).
+ *  - `stream` is a cudaStream_t passed as void* (NULL = the legacy default stream). Every call
+ *    only enqueues work on `stream` and returns without synchronising.
+ *  - The return value reports what the host can see: bad arguments (VARRATE_ERR_ARG), a workspace
+ *    that is too small (VARRATE_ERR_WORKSPACE), an unsupported shape (VARRATE_ERR_UNSUPPORTED) or
+ *    a failed launch (VARRATE_ERR_CUDA). Nothing is enqueued when the return value is negative.
+ *  - Outcomes that depend on the data are written by the kernels to `*dev_status` (one int32 in
+ *    device memory). Kernels only raise it: a warning (VARRATE_FLOOR_BINDS) replaces 0, an error
+ *    (negative) replaces anything larger. The caller zeroes it before a sequence of calls and
+ *    reads it after synchronising.
+ *  - dtype VARRATE_BF16: keys, values, queries, bases and packed coefficients are bfloat16 and all
+ *    arithmetic accumulates in fp32. dtype VARRATE_F32: all of them are fp32. Salience is fp32 in
+ *    both cases.
+ *  - Limits: head_dim == 128, 1 <= group <= 8, 1 <= window and group * window <= 256,
+ *    window <= n_ctx < 2^31, 1 <= r_min <= head_dim, pool_len odd in [1, 31],
+ *    0 < budget_frac <= 1.
+ *
+ * Notation: B = batch (sequences), L = n_layers, G = n_kv_heads, H = G * group query heads,
+ * d = head_dim, N = n_ctx, w = window. The exact set is the last w tokens [N - w, N) (kept at
+ * full rank d); the coded set is [0, N - w).
+ */
+#ifndef VARRATE_H
+#define VARRATE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  VARRATE_OK = 0,
+  VARRATE_FLOOR_BINDS = 1,       /* warning: budget below r_min * |C|; every coded token at r_min */
+  VARRATE_ERR_ARG = -1,          /* invalid argument (null pointer, size out of range) */
+  VARRATE_ERR_WORKSPACE = -2,    /* ws_bytes smaller than varrate_workspace_bytes() */
+  VARRATE_ERR_CUDA = -3,         /* a CUDA launch or runtime call failed */
+  VARRATE_ERR_TIMEOUT = -4,      /* a bounded device-side wait gave up */
+  VARRATE_ERR_UNSUPPORTED = -5,  /* a shape outside the limits above */
+  VARRATE_ERR_CORRUPT = -6       /* rank or layout table outside its valid range */
+} varrate_status;
+
+typedef enum { VARRATE_F32 = 0, VARRATE_BF16 = 1 } varrate_dtype;
+
+/* Allocation mode: salience-driven water-filling (Sec. 3.2, Eq. 4) or the uniform-rank "flat"
+ * ablation (every coded token at the same rank; the constant-salience limit of Eq. 4). */
+typedef enum { VARRATE_SALIENCE = 0, VARRATE_UNIFORM = 1 } varrate_mode;
+
+/* Problem statement (Sec. 3.1 "Attention and the KV cache", "Budget"; Sec. 4.1). r_max is head_dim. */
+typedef struct {
+  int32_t n_layers;     /* L */
+  int32_t n_kv_heads;   /* G */
+  int32_t group;        /* query heads per KV head (GQA) */
+  int32_t head_dim;     /* d (must be 128) */
+  int64_t n_ctx;        /* N, cached tokens per sequence */
+  int32_t batch;        /* B, independent sequences */
+  int32_t r_min;        /* rank floor (Eq. 4) */
+  double budget_frac;   /* kappa: fraction of the full cache kept (Eq. 3) */
+  int32_t window;       /* w = observation window = exact recent window */
+  int32_t pool_len;     /* moving-average length of the salience (5 in SnapKV) */
+  int32_t dtype;        /* varrate_dtype */
+  int32_t mode;         /* varrate_mode */
+} varrate_config;
+
+/* Packed variable-rank cache (all device pointers, caller-owned).
+ *
+ * For each (sequence b, layer l) one bucket table, shared by every KV head and by K and V, groups
+ * the tokens by rank. With n_r tokens of rank r and n8_r = n_r rounded up to a multiple of 8:
+ *   bucket_base[r_min] = 0, bucket_base[r + 1] = bucket_base[r] + r * n8_r,
+ * and coefficient j (< r_t) of token t of stream (b, l, g, kv) sits at element
+ *   coef[(((b * L + l) * G + g) * 2 + kv) * cap_elems + bucket_base[r_t] + j * n8_{r_t} + pos[t]]
+ * (coefficient-major inside a bucket: one coefficient of consecutive tokens is contiguous).
+ * Padding slots pos in [n_r, n8_r) hold zeros. kv = 0 is K, 1 is V. */
+typedef struct {
+  void* coef;             /* [B][L][G][2][cap_elems] dtype */
+  int32_t* bucket_count;  /* [B][L][d + 1]  n_r (0 for r < r_min) */
+  int64_t* bucket_base;   /* [B][L][d + 2]  element offset of bucket r (0 for r <= r_min) */
+  int32_t* perm;          /* [B][L][N] bucketed slot -> token (buckets in increasing rank, stable) */
+  int32_t* pos;           /* [B][L][N] token -> position inside its bucket */
+  uint8_t* ranks;         /* [B][L][N] rank of every token (exact set at d) */
+  int64_t cap_elems;      /* elements per stream, >= varrate_packed_cap_elems() */
+} varrate_packed;
+
+/* Which call a workspace is sized for. */
+typedef enum {
+  VARRATE_CALL_SALIENCE = 0,
+  VARRATE_CALL_PACK = 1,
+  VARRATE_CALL_ENCODE = 2,
+  VARRATE_CALL_DECODE = 3
+} varrate_call;
+
+/* Library version (major * 10000 + minor * 100 + patch). */
+int32_t varrate_version(void);
+
+/* Readable name of a status code; never NULL. */
+const char* varrate_status_string(int32_t status);
+
+/* Validates a configuration against the limits above; VARRATE_OK or the error it would cause. */
+varrate_status varrate_check_config(const varrate_config* cfg);
+
+/* Coded budget B_c of one (sequence, layer) in per-head rank units: Eq. 3 (Sec. 3.1) with
+ * D -> d and n_ref = w, i.e. floor(budget_frac * (N * d)) - w * d, the product in double.
+ * Returns INT64_MIN if cfg is invalid. */
+int64_t varrate_coded_budget(const varrate_config* cfg);
+
+/* Upper bound on the packed length of one stream, independent of the data:
+ * max(B_c, r_min * (N - w)) + w * d + 7 * sum_{r = r_min..d} r. Returns -1 if cfg is invalid. */
+int64_t varrate_packed_cap_elems(const varrate_config* cfg);
+
+/* Bytes of device workspace a call needs (0 is a valid answer). Returns 0 if cfg is invalid. */
+size_t varrate_workspace_bytes(const varrate_config* cfg, int32_t which_call);
+
+/* Step 1 — salience (Sec. 3.2, Eq. salience, and SnapKV's length-pool_len moving average).
+ *   q_win   [B][L][w][H][d]  queries of the last w tokens (window query q is at position N - w + q)
+ *   k       [B][L][G][N][d]  keys; query head h reads KV head h / group
+ *   sal_out [B][L][N - w]    fp32: s'_t = pooled mean over the w queries and H heads of the
+ *                            causal softmax weight alpha_{q,t} = softmax_{u <= p}(<q,k_u>/sqrt(d))
+ *   ws      workspace of at least varrate_workspace_bytes(cfg, VARRATE_CALL_SALIENCE) bytes. */
+varrate_status varrate_salience(const varrate_config* cfg, const void* q_win, const void* k,
+                                float* sal_out, void* ws, size_t ws_bytes, void* stream);
+
+/* Step 2 — rank allocation (Sec. 3.2, Eq. 4 and Algorithm 1's water level), per (b, l):
+ * min-max normalise sal over the coded set in IEEE fp32 (s_hat = (s - min) / (max - min); 1 if
+ * max == min or mode is UNIFORM), then rank_t = r_max if x_t >= r_max else max(r_min, floor(x_t))
+ * with x_t = fl(fl(lambda * s_hat_t) + r_min), lambda the largest fp32 value whose ranks sum to at
+ * most B_c. If r_min * |C| > B_c every coded token gets r_min and *dev_status is raised to
+ * VARRATE_FLOOR_BINDS; if B_c >= d * |C| every token gets d. The exact set gets d.
+ *   sal          [B][L][N - w] fp32 (e.g. from varrate_salience; ignored in UNIFORM mode, may be NULL)
+ *   ranks        [B][L][N] uint8 out
+ *   realized_sum [B][L] int64 out: sum of the coded ranks (<= B_c unless FLOOR_BINDS); may be NULL
+ * The result is a deterministic function of the fp32 input bits. */
+varrate_status varrate_allocate(const varrate_config* cfg, const float* sal, uint8_t* ranks,
+                                int64_t* realized_sum, int32_t* dev_status, void* stream);
+
+/* Step 3 — projection and packing (Algorithm 1's projection; Eq. 5 with the anchor mean at 0):
+ * builds the bucket tables of `out` from `out->ranks` (which the caller fills, e.g. with
+ * varrate_allocate), then writes c_t = U_{g} x_t truncated to r_t for every stream.
+ *   k, v        [B][L][G][N][d]
+ *   basis_k/_v  [L][G][d][d]  row j = basis vector j (ordered by decreasing singular value)
+ * A rank outside [r_min, d] in out->ranks raises VARRATE_ERR_CORRUPT and leaves coef undefined. */
+varrate_status varrate_pack(const varrate_config* cfg, const void* k, const void* v,
+                            const void* basis_k, const void* basis_v, varrate_packed* out,
+                            int32_t* dev_status, void* ws, size_t ws_bytes, void* stream);
+
+/* Steps 1-3 for every (b, l): varrate_salience, varrate_allocate and varrate_pack in one call.
+ * sal_out and realized_sum may be NULL (then kept in the workspace). */
+varrate_status varrate_encode(const varrate_config* cfg, const void* q_win, const void* k,
+                              const void* v, const void* basis_k, const void* basis_v,
+                              float* sal_out, varrate_packed* out, int64_t* realized_sum,
+                              int32_t* dev_status, void* ws, size_t ws_bytes, void* stream);
+
+/* Step 4 — decode attention on the packed coefficients of one layer (attention of Sec. 3.1 over
+ * the cache of Eq. 5, without rebuilding K or V): per query head h of KV head g,
+ *   q~ = U_K q;  score_t = q~[:r_t] . c^K_t[:r_t] / sqrt(d);  alpha = softmax over all N tokens
+ *   (and the n_tail exact tail tokens);  o = U_V^T sum_t alpha_t c^V_t[:r_t] + sum_tail alpha v.
+ *   q       [B][H][d]  one query per head per sequence
+ *   tail_k/_v [B][G][n_tail][d] uncompressed tokens appended after the cache (may be NULL if
+ *           n_tail == 0)
+ *   out     [B][H][d]  dtype
+ *   ws      at least varrate_workspace_bytes(cfg, VARRATE_CALL_DECODE) bytes. */
+varrate_status varrate_decode_attn(const varrate_config* cfg, const varrate_packed* cache,
+                                   const void* basis_k, const void* basis_v, const void* q,
+                                   int32_t layer, const void* tail_k, const void* tail_v,
+                                   int32_t n_tail, void* out, int32_t* dev_status, void* ws,
+                                   size_t ws_bytes, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* VARRATE_H */

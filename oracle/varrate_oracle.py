@@ -312,12 +312,14 @@ def attention(q: np.ndarray, k: np.ndarray, v: np.ndarray) -> np.ndarray:
     return out
 
 
-def decode_coef(q, coef_k, coef_v, ranks, basis_k, basis_v) -> np.ndarray:
+def decode_coef(q, coef_k, coef_v, ranks, basis_k, basis_v, tail_k=None, tail_v=None):
     """Decode attention computed on the coefficients (route i).
 
     q [H][d]; coef_k, coef_v [G][N][d] full coefficients (truncated here by ranks);
-    basis_k, basis_v [G][d][d]. Per head: q~ = U_K q; score_t = q~[:r_t] . c^K_t[:r_t] / sqrt(d);
-    alpha = softmax over all N tokens; o~ = sum_t alpha_t (m_t * c^V_t); o = U_V^T o~.
+    basis_k, basis_v [G][d][d]; optional tail_k, tail_v [G][n_tail][d] exact tokens appended after
+    the cache (the recent window kept exact, Sec. 3.1 "Residual codec"). Per head:
+    q~ = U_K q; score_t = q~[:r_t] . c^K_t[:r_t] / sqrt(d) (tail: q . k / sqrt(d)); alpha = softmax
+    over all N (+ n_tail) tokens; o = U_V^T sum_t alpha_t (m_t * c^V_t) + sum_tail alpha v.
     Equal to attention over the reconstructed cache because U_K^T is the inverse rotation."""
     q = np.asarray(q, dtype=np.float64)
     H, d = q.shape
@@ -332,18 +334,30 @@ def decode_coef(q, coef_k, coef_v, ranks, basis_k, basis_v) -> np.ndarray:
         ck = truncate(np.asarray(coef_k[g], dtype=np.float64), ranks)
         cv = truncate(np.asarray(coef_v[g], dtype=np.float64), ranks)
         sc = ck @ qt / math.sqrt(d)
-        a = np.exp(sc - sc.max())
-        a /= a.sum()
-        out[h] = uv.T @ (a @ cv)
+        if tail_k is not None and len(tail_k[g]):
+            tk = np.asarray(tail_k[g], dtype=np.float64)
+            tv = np.asarray(tail_v[g], dtype=np.float64)
+            st = tk @ q[h] / math.sqrt(d)
+        else:
+            tv = np.zeros((0, d))
+            st = np.zeros(0)
+        m = max(sc.max(), st.max() if st.size else -np.inf)
+        a = np.exp(sc - m)
+        at = np.exp(st - m)
+        z = a.sum() + at.sum()
+        out[h] = (uv.T @ (a @ cv) + at @ tv) / z
     return out
 
 
-def decode_recon(q, coef_k, coef_v, ranks, basis_k, basis_v) -> np.ndarray:
-    """Decode attention on the reconstructed cache (route ii): rebuild k_hat, v_hat by Eq. 5 and
-    run plain attention over them (the paper's reconstruct-in-place decode)."""
+def decode_recon(q, coef_k, coef_v, ranks, basis_k, basis_v, tail_k=None, tail_v=None):
+    """Decode attention on the reconstructed cache (route ii): rebuild k_hat, v_hat by Eq. 5,
+    append the exact tail tokens and run plain attention (the paper's reconstruct-in-place decode)."""
     G = coef_k.shape[0]
     kh = np.stack([reconstruct(coef_k[g], ranks, basis_k[g]) for g in range(G)])
     vh = np.stack([reconstruct(coef_v[g], ranks, basis_v[g]) for g in range(G)])
+    if tail_k is not None:
+        kh = np.concatenate([kh, np.asarray(tail_k, dtype=np.float64)], axis=1)
+        vh = np.concatenate([vh, np.asarray(tail_v, dtype=np.float64)], axis=1)
     return attention(q, kh, vh)
 
 

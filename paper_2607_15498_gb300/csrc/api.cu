@@ -1,0 +1,209 @@
+// C ABI of the VarRate hot path (declared in include/varrate.h): argument validation, workspace
+// carving and kernel launches. No device memory is allocated here.
+#include <math.h>
+#include <stdint.h>
+
+#include "common.cuh"
+#include "kernels.h"
+
+using vr::Shape;
+
+namespace {
+
+constexpr int32_t kVersion = 1 * 10000 + 0 * 100 + 0;
+
+bool valid_dtype(int32_t d) { return d == VARRATE_F32 || d == VARRATE_BF16; }
+
+varrate_status check(const varrate_config* c) {
+  if (c == nullptr) return VARRATE_ERR_ARG;
+  if (c->n_layers < 1 || c->n_kv_heads < 1 || c->group < 1 || c->batch < 1 || c->window < 1 ||
+      c->n_ctx < 1 || c->r_min < 1 || !valid_dtype(c->dtype) ||
+      (c->mode != VARRATE_SALIENCE && c->mode != VARRATE_UNIFORM))
+    return VARRATE_ERR_ARG;
+  if (!(c->budget_frac > 0.0) || !(c->budget_frac <= 1.0)) return VARRATE_ERR_ARG;
+  if (c->window > c->n_ctx || c->n_ctx >= (int64_t(1) << 31)) return VARRATE_ERR_ARG;
+  if (c->pool_len < 1 || c->pool_len > 31 || (c->pool_len % 2) == 0) return VARRATE_ERR_ARG;
+  if (c->head_dim != vr::kHeadDim) return VARRATE_ERR_UNSUPPORTED;
+  if (c->r_min > c->head_dim) return VARRATE_ERR_ARG;
+  if (c->group > 8 || (int64_t)c->group * c->window > 256) return VARRATE_ERR_UNSUPPORTED;
+  return VARRATE_OK;
+}
+
+int64_t coded_budget(const varrate_config* c) {
+  return (int64_t)floor(c->budget_frac * (double)(c->n_ctx * (int64_t)c->head_dim)) -
+         (int64_t)c->window * c->head_dim;
+}
+
+int64_t cap_elems(const varrate_config* c) {
+  const int64_t n_coded = c->n_ctx - c->window;
+  int64_t coded = coded_budget(c);
+  if ((int64_t)c->r_min * n_coded > coded) coded = (int64_t)c->r_min * n_coded;
+  if (coded < 0) coded = 0;
+  int64_t pads = 0;
+  for (int r = c->r_min; r <= c->head_dim; ++r) pads += 7 * r;
+  const int64_t cap = coded + (int64_t)c->window * c->head_dim + pads;
+  return (cap + 7) & ~int64_t(7);
+}
+
+Shape make_shape(const varrate_config* c, int64_t cap) {
+  Shape s;
+  s.B = c->batch; s.L = c->n_layers; s.G = c->n_kv_heads; s.grp = c->group;
+  s.H = c->n_kv_heads * c->group; s.d = c->head_dim; s.w = c->window; s.pool = c->pool_len;
+  s.r_min = c->r_min; s.r_max = c->head_dim; s.dtype = c->dtype; s.mode = c->mode;
+  s.N = c->n_ctx; s.n_coded = c->n_ctx - c->window; s.Bc = coded_budget(c); s.cap = cap;
+  return s;
+}
+
+int num_sms() {
+  static int cached[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 148;
+  if (cached[dev] == 0) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 148;
+    cached[dev] = n;
+  }
+  return cached[dev];
+}
+
+size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+size_t ws_bytes(const varrate_config* c, int32_t which) {
+  const Shape s = make_shape(c, cap_elems(c));
+  const int sms = num_sms();
+  switch (which) {
+    case VARRATE_CALL_SALIENCE: return vr::salience_ws_bytes(s, sms);
+    case VARRATE_CALL_PACK: return 0;
+    case VARRATE_CALL_ENCODE:
+      return vr::salience_ws_bytes(s, sms) + align256((size_t)s.B * s.L * s.n_coded * sizeof(float)) +
+             align256((size_t)s.B * s.L * sizeof(int64_t));
+    case VARRATE_CALL_DECODE: return vr::decode_ws_bytes(s, sms);
+    default: return 0;
+  }
+}
+
+varrate_status launched() {
+  return cudaGetLastError() == cudaSuccess ? VARRATE_OK : VARRATE_ERR_CUDA;
+}
+
+bool packed_ok(const varrate_config* c, const varrate_packed* p) {
+  return p && p->coef && p->bucket_count && p->bucket_base && p->perm && p->pos && p->ranks &&
+         p->cap_elems >= cap_elems(c) && (p->cap_elems % 8) == 0;
+}
+
+}  // namespace
+
+extern "C" {
+
+int32_t varrate_version(void) { return kVersion; }
+
+const char* varrate_status_string(int32_t st) {
+  switch (st) {
+    case VARRATE_OK: return "ok";
+    case VARRATE_FLOOR_BINDS: return "budget below the rank floor: every coded token at r_min";
+    case VARRATE_ERR_ARG: return "invalid argument";
+    case VARRATE_ERR_WORKSPACE: return "workspace too small";
+    case VARRATE_ERR_CUDA: return "CUDA launch or runtime error";
+    case VARRATE_ERR_TIMEOUT: return "bounded device wait timed out";
+    case VARRATE_ERR_UNSUPPORTED: return "unsupported shape";
+    case VARRATE_ERR_CORRUPT: return "rank or layout table out of range";
+    default: return "unknown status";
+  }
+}
+
+varrate_status varrate_check_config(const varrate_config* cfg) { return check(cfg); }
+
+int64_t varrate_coded_budget(const varrate_config* cfg) {
+  return check(cfg) == VARRATE_OK ? coded_budget(cfg) : INT64_MIN;
+}
+
+int64_t varrate_packed_cap_elems(const varrate_config* cfg) {
+  return check(cfg) == VARRATE_OK ? cap_elems(cfg) : -1;
+}
+
+size_t varrate_workspace_bytes(const varrate_config* cfg, int32_t which_call) {
+  return check(cfg) == VARRATE_OK ? ws_bytes(cfg, which_call) : 0;
+}
+
+varrate_status varrate_salience(const varrate_config* cfg, const void* q_win, const void* k,
+                                float* sal_out, void* ws, size_t ws_bytes_, void* stream) {
+  varrate_status st = check(cfg);
+  if (st != VARRATE_OK) return st;
+  const bool empty = cfg->n_ctx == cfg->window;   // no coded token: nothing to score
+  if (!empty && (!q_win || !k || !sal_out)) return VARRATE_ERR_ARG;
+  if (cfg->mode == VARRATE_UNIFORM) return VARRATE_ERR_ARG;
+  const size_t need = ws_bytes(cfg, VARRATE_CALL_SALIENCE);
+  if (ws_bytes_ < need || (need > 0 && ws == nullptr)) return VARRATE_ERR_WORKSPACE;
+  const Shape s = make_shape(cfg, cap_elems(cfg));
+  vr::launch_salience(s, q_win, k, sal_out, ws, num_sms(), (cudaStream_t)stream);
+  return launched();
+}
+
+varrate_status varrate_allocate(const varrate_config* cfg, const float* sal, uint8_t* ranks,
+                                int64_t* realized_sum, int32_t* dev_status, void* stream) {
+  varrate_status st = check(cfg);
+  if (st != VARRATE_OK) return st;
+  if (!ranks || (cfg->mode == VARRATE_SALIENCE && !sal && cfg->n_ctx > cfg->window))
+    return VARRATE_ERR_ARG;
+  const Shape s = make_shape(cfg, cap_elems(cfg));
+  vr::launch_allocate(s, sal, ranks, realized_sum, dev_status, (cudaStream_t)stream);
+  return launched();
+}
+
+varrate_status varrate_pack(const varrate_config* cfg, const void* k, const void* v,
+                            const void* basis_k, const void* basis_v, varrate_packed* out,
+                            int32_t* dev_status, void* ws, size_t ws_bytes_, void* stream) {
+  (void)ws; (void)ws_bytes_;
+  varrate_status st = check(cfg);
+  if (st != VARRATE_OK) return st;
+  if (!k || !v || !basis_k || !basis_v || !packed_ok(cfg, out)) return VARRATE_ERR_ARG;
+  const Shape s = make_shape(cfg, out->cap_elems);
+  vr::launch_pack(s, k, v, basis_k, basis_v, *out, dev_status, num_sms(), (cudaStream_t)stream);
+  return launched();
+}
+
+varrate_status varrate_encode(const varrate_config* cfg, const void* q_win, const void* k,
+                              const void* v, const void* basis_k, const void* basis_v,
+                              float* sal_out, varrate_packed* out, int64_t* realized_sum,
+                              int32_t* dev_status, void* ws, size_t ws_bytes_, void* stream) {
+  varrate_status st = check(cfg);
+  if (st != VARRATE_OK) return st;
+  if (!k || !v || !basis_k || !basis_v || !packed_ok(cfg, out)) return VARRATE_ERR_ARG;
+  if (cfg->mode == VARRATE_SALIENCE && !q_win && cfg->n_ctx > cfg->window) return VARRATE_ERR_ARG;
+  const size_t need = ws_bytes(cfg, VARRATE_CALL_ENCODE);
+  if (ws_bytes_ < need || ws == nullptr) return VARRATE_ERR_WORKSPACE;
+  const Shape s = make_shape(cfg, out->cap_elems);
+  const int sms = num_sms();
+  cudaStream_t cs = (cudaStream_t)stream;
+  char* w = static_cast<char*>(ws);
+  const size_t sal_ws = vr::salience_ws_bytes(s, sms);
+  float* sal = sal_out ? sal_out : reinterpret_cast<float*>(w + sal_ws);
+  int64_t* realized = realized_sum
+      ? realized_sum
+      : reinterpret_cast<int64_t*>(w + sal_ws + align256((size_t)s.B * s.L * s.n_coded * sizeof(float)));
+  if (cfg->mode == VARRATE_SALIENCE) vr::launch_salience(s, q_win, k, sal, w, sms, cs);
+  vr::launch_allocate(s, sal, out->ranks, realized, dev_status, cs);
+  vr::launch_pack(s, k, v, basis_k, basis_v, *out, dev_status, sms, cs);
+  return launched();
+}
+
+varrate_status varrate_decode_attn(const varrate_config* cfg, const varrate_packed* cache,
+                                   const void* basis_k, const void* basis_v, const void* q,
+                                   int32_t layer, const void* tail_k, const void* tail_v,
+                                   int32_t n_tail, void* out, int32_t* dev_status, void* ws,
+                                   size_t ws_bytes_, void* stream) {
+  varrate_status st = check(cfg);
+  if (st != VARRATE_OK) return st;
+  if (!packed_ok(cfg, cache) || !basis_k || !basis_v || !q || !out) return VARRATE_ERR_ARG;
+  if (layer < 0 || layer >= cfg->n_layers || n_tail < 0) return VARRATE_ERR_ARG;
+  if (n_tail > 4096) return VARRATE_ERR_UNSUPPORTED;
+  if (n_tail > 0 && (!tail_k || !tail_v)) return VARRATE_ERR_ARG;
+  const size_t need = ws_bytes(cfg, VARRATE_CALL_DECODE);
+  if (ws_bytes_ < need || ws == nullptr) return VARRATE_ERR_WORKSPACE;
+  const Shape s = make_shape(cfg, cache->cap_elems);
+  vr::launch_decode(s, *cache, basis_k, basis_v, q, layer, tail_k, tail_v, n_tail, out, dev_status,
+                    ws, num_sms(), (cudaStream_t)stream);
+  return launched();
+}
+
+}  // extern "C"

@@ -1,0 +1,43 @@
+// Host-side launchers of the VarRate kernels (internal; the public ABI is include/varrate.h).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "common.cuh"
+
+namespace vr {
+
+// ---- step 1: salience
+struct SalPlan {
+  int n_rb;          // row blocks of 128 window rows per KV head
+  int n_chunks;      // token chunks of pass 1
+  int64_t chunk;
+  int n_chunks2;     // token chunks of pass 2
+  int64_t chunk2;
+};
+SalPlan salience_plan(const Shape& s, int num_sms);
+size_t salience_ws_bytes(const Shape& s, int num_sms);
+// Returns the number of kernels launched.
+int launch_salience(const Shape& s, const void* q_win, const void* k, float* sal_out, void* ws,
+                    int num_sms, cudaStream_t st);
+
+// ---- step 2: allocation
+int launch_allocate(const Shape& s, const float* sal, uint8_t* ranks, int64_t* realized,
+                    int32_t* dev_status, cudaStream_t st);
+
+// ---- step 3: tables + projection
+int launch_pack(const Shape& s, const void* k, const void* v, const void* basis_k,
+                const void* basis_v, const varrate_packed& out, int32_t* dev_status,
+                int num_sms, cudaStream_t st);
+
+// ---- step 4: decode attention
+int decode_splits(const Shape& s, int num_sms);
+size_t decode_ws_bytes(const Shape& s, int num_sms);
+int launch_decode(const Shape& s, const varrate_packed& cache, const void* basis_k,
+                  const void* basis_v, const void* q, int layer, const void* tail_k,
+                  const void* tail_v, int n_tail, void* out, int32_t* dev_status, void* ws,
+                  int num_sms, cudaStream_t st);
+
+}  // namespace vr

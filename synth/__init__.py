@@ -212,3 +212,34 @@ def basis_tensors(wl: Workload, layer: int, device="cpu", out_dtype=None):
     uk, uv = bases(wl, layer)
     return (torch.tensor(uk, dtype=torch.float64).to(dt).to(device),
             torch.tensor(uv, dtype=torch.float64).to(dt).to(device))
+
+
+def stack_inputs(wl: Workload, device="cpu", out_dtype=None, batch_index: int = 0):
+    """All encode inputs of a workload, stacked in the library's layouts:
+    k, v [B][L][G][N][d]; q_win [B][L][w][H][d]; basis_k, basis_v [L][G][d][d]."""
+    dt = out_dtype or torch_dtype(wl)
+    B, L, G, N, d = wl.batch, wl.n_layers, wl.n_kv_heads, wl.n_ctx, wl.head_dim
+    k = torch.empty((B, L, G, N, d), dtype=dt, device=device)
+    v = torch.empty_like(k)
+    qw = torch.empty((B, L, wl.window, wl.n_q_heads, d), dtype=dt, device=device)
+    for b in range(B):
+        for l in range(L):
+            kk, vv = layer_kv(wl, b, l, device=device, out_dtype=dt)
+            k[b, l] = kk
+            v[b, l] = vv
+            qw[b, l] = window_queries(wl, b, l, device=device, out_dtype=dt, batch_index=batch_index)
+    bk = torch.empty((L, G, d, d), dtype=dt, device=device)
+    bv = torch.empty_like(bk)
+    for l in range(L):
+        a, c = basis_tensors(wl, l, device=device, out_dtype=dt)
+        bk[l] = a
+        bv[l] = c
+    return k, v, qw, bk, bv
+
+
+def stack_decode_queries(wl: Workload, layer: int, n_steps: int, device="cpu", out_dtype=None,
+                         batch_index: int = 0) -> torch.Tensor:
+    """Decode queries of every sequence for one layer: [n_steps][B][H][d]."""
+    qs = [decode_queries(wl, b, layer, n_steps, device=device, out_dtype=out_dtype,
+                         batch_index=batch_index) for b in range(wl.batch)]
+    return torch.stack(qs, dim=1)

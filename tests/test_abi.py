@@ -1,0 +1,133 @@
+"""Host-side checks of the C ABI (no GPU needed): the library loads, exports every function that
+include/varrate.h declares, and its host-only functions (budget, sizing, validation) agree with
+the oracle and reject bad arguments before touching a device."""
+import json
+import os
+import re
+import subprocess
+
+import pytest
+
+import oracle as O
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "varrate.h")
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(varrate_\w+)\s*\(", text)))
+
+
+def test_header_declares_the_hot_path():
+    names = declared_functions()
+    for must in ("varrate_encode", "varrate_allocate", "varrate_pack", "varrate_decode_attn",
+                 "varrate_salience"):
+        assert must in names
+
+
+def test_library_exports_every_declared_symbol(vlib):
+    lib = vlib.lib()
+    out = subprocess.run(["nm", "-D", "--defined-only", vlib.LIB_PATH], capture_output=True,
+                         text=True).stdout
+    exported = set(re.findall(r"\bT (varrate_\w+)", out))
+    for name in declared_functions():
+        assert name in exported, name
+        assert hasattr(lib, name)
+    assert set(vlib.EXPORTED) == set(declared_functions())
+
+
+def test_version_and_status_strings(vlib):
+    assert vlib.varrate_version() >= 10000
+    for code in (0, 1, -1, -2, -3, -4, -5, -6):
+        assert vlib.status_string(code) and vlib.status_string(code) != "unknown status"
+    assert vlib.status_string(12345) == "unknown status"
+
+
+def test_coded_budget_matches_oracle_golden(vlib):
+    with open(os.path.join(ROOT, "tests", "golden", "budgets.json")) as f:
+        for c in json.load(f)["cases"]:
+            cfg = vlib.make_config(1, 1, 1, c["n_ctx"], budget_frac=c["budget_frac"],
+                                   window=c["window"], head_dim=c["head_dim"])
+            assert vlib.varrate_coded_budget(cfg) == c["B_c"] == O.coded_budget(
+                c["n_ctx"], c["head_dim"], c["window"], c["budget_frac"])
+
+
+@pytest.mark.parametrize("n_ctx,w,kappa,rmin", [(2048, 32, 0.2, 16), (32768, 32, 0.1, 16),
+                                                (32768, 32, 1.0, 16), (100, 100, 0.5, 1),
+                                                (1037, 5, 0.33, 7)])
+def test_cap_bounds_oracle(vlib, n_ctx, w, kappa, rmin):
+    cfg = vlib.make_config(1, 1, 1, n_ctx, budget_frac=kappa, window=w, r_min=rmin)
+    cap = vlib.varrate_packed_cap_elems(cfg)
+    assert cap % 8 == 0
+    assert cap >= O.packed_cap_elems(n_ctx, 128, w, kappa, rmin)
+
+
+@pytest.mark.parametrize("field,value,want", [
+    ("head_dim", 64, -5), ("group", 9, -5), ("window", 0, -1), ("r_min", 0, -1),
+    ("r_min", 129, -1), ("budget_frac", 0.0, -1), ("budget_frac", 1.5, -1), ("pool_len", 4, -1),
+    ("dtype", 7, -1), ("mode", 3, -1), ("n_ctx", 16, -1), ("batch", 0, -1)])
+def test_check_config_rejects(vlib, field, value, want):
+    cfg = vlib.make_config(2, 8, 4, 32768)
+    assert vlib.varrate_check_config(cfg) == 0
+    setattr(cfg, field, value)
+    assert vlib.varrate_check_config(cfg) == want
+    assert vlib.varrate_coded_budget(cfg) == -(2 ** 63)
+    assert vlib.varrate_packed_cap_elems(cfg) == -1
+    assert vlib.varrate_workspace_bytes(cfg, vlib.CALL_ENCODE) == 0
+
+
+def test_group_window_product_limit(vlib):
+    cfg = vlib.make_config(1, 2, 8, 4096, window=32)
+    assert vlib.varrate_check_config(cfg) == 0
+    cfg.window = 33
+    assert vlib.varrate_check_config(cfg) == vlib.ERR_UNSUPPORTED
+
+
+def test_workspace_sizes_positive(vlib):
+    cfg = vlib.make_config(32, 8, 4, 32768, batch=8)
+    for which in (vlib.CALL_SALIENCE, vlib.CALL_ENCODE, vlib.CALL_DECODE):
+        assert vlib.varrate_workspace_bytes(cfg, which) > 0
+    assert vlib.varrate_workspace_bytes(cfg, vlib.CALL_PACK) == 0
+
+
+def test_null_arguments_rejected_on_host(vlib):
+    cfg = vlib.make_config(1, 1, 4, 2048, dtype=vlib.F32)
+    L = vlib.lib()
+    assert L.varrate_salience(vlib.ctypes.byref(cfg), None, None, None, None, 0, None) == vlib.ERR_ARG
+    assert L.varrate_allocate(vlib.ctypes.byref(cfg), None, None, None, None, None) == vlib.ERR_ARG
+    p = vlib.varrate_packed()
+    assert L.varrate_pack(vlib.ctypes.byref(cfg), 1, 1, 1, 1, vlib.ctypes.byref(p), None, None, 0,
+                          None) == vlib.ERR_ARG
+    assert L.varrate_encode(vlib.ctypes.byref(cfg), 1, 1, 1, 1, 1, None, vlib.ctypes.byref(p), None,
+                            None, None, 0, None) == vlib.ERR_ARG
+    assert L.varrate_decode_attn(vlib.ctypes.byref(cfg), vlib.ctypes.byref(p), 1, 1, 1, 0, None,
+                                 None, 0, 1, None, None, 0, None) == vlib.ERR_ARG
+
+
+def test_small_workspace_and_bad_layer_rejected_on_host(vlib):
+    cfg = vlib.make_config(2, 1, 4, 2048, dtype=vlib.F32)
+    L = vlib.lib()
+    cap = vlib.varrate_packed_cap_elems(cfg)
+    p = vlib.varrate_packed(1, 1, 1, 1, 1, 1, cap)
+    assert L.varrate_decode_attn(vlib.ctypes.byref(cfg), vlib.ctypes.byref(p), 1, 1, 1, 2, None,
+                                 None, 0, 1, None, 1, 1 << 40, None) == vlib.ERR_ARG
+    assert L.varrate_decode_attn(vlib.ctypes.byref(cfg), vlib.ctypes.byref(p), 1, 1, 1, 0, None,
+                                 None, 0, 1, None, 1, 16, None) == vlib.ERR_WORKSPACE
+    assert L.varrate_decode_attn(vlib.ctypes.byref(cfg), vlib.ctypes.byref(p), 1, 1, 1, 0, None,
+                                 None, 5000, 1, None, 1, 1 << 40, None) == vlib.ERR_UNSUPPORTED
+    p.cap_elems = cap - 8
+    assert L.varrate_decode_attn(vlib.ctypes.byref(cfg), vlib.ctypes.byref(p), 1, 1, 1, 0, None,
+                                 None, 0, 1, None, 1, 1 << 40, None) == vlib.ERR_ARG
+    assert L.varrate_encode(vlib.ctypes.byref(cfg), 1, 1, 1, 1, 1, None,
+                            vlib.ctypes.byref(vlib.varrate_packed(1, 1, 1, 1, 1, 1, cap)), None,
+                            None, 1, 8, None) == vlib.ERR_WORKSPACE
+
+
+def test_binding_fails_loudly_without_library(tmp_path, monkeypatch):
+    from paper_2607_15498_gb300 import varrate as V
+    monkeypatch.setattr(V, "_lib", None)
+    monkeypatch.setattr(V, "LIB_PATH", str(tmp_path / "missing.so"))
+    with pytest.raises(RuntimeError, match="no CPU fallback"):
+        V.lib()

@@ -317,6 +317,25 @@ def test_decode_routes_agree_and_full_rank_is_exact():
     np.testing.assert_allclose(full, _sdpa_attention(q, k, v), atol=1e-10)
 
 
+def test_decode_with_exact_tail():
+    wl = synth.workload("tiny", n_ctx=200, window=8, n_kv_heads=2)
+    k, v = synth.layer_kv(wl, 0, 0, out_dtype=torch.float64)
+    k, v = k.numpy(), v.numpy()
+    uk, uv = synth.bases(wl, 0)
+    rng = np.random.default_rng(11)
+    q = rng.standard_normal((wl.n_q_heads, wl.head_dim))
+    tk = rng.standard_normal((2, 5, wl.head_dim))
+    tv = rng.standard_normal((2, 5, wl.head_dim))
+    ck = np.stack([O.project(k[g], uk[g]) for g in range(2)])
+    cv = np.stack([O.project(v[g], uv[g]) for g in range(2)])
+    ranks = rng.integers(16, 129, size=200)
+    a = O.decode_coef(q, ck, cv, ranks, uk, uv, tk, tv)
+    np.testing.assert_allclose(a, O.decode_recon(q, ck, cv, ranks, uk, uv, tk, tv), atol=1e-10)
+    full = O.decode_coef(q, ck, cv, np.full(200, 128), uk, uv, tk, tv)
+    want = _sdpa_attention(q, np.concatenate([k, tk], 1), np.concatenate([v, tv], 1))
+    np.testing.assert_allclose(full, want, atol=1e-10)
+
+
 def test_decode_single_token_and_flat_scores():
     d = 16
     rng = np.random.default_rng(8)
