@@ -176,6 +176,25 @@ varrate_status varrate_decode_attn(const varrate_config* cfg, const varrate_pack
                                    int32_t n_tail, void* out, int32_t* dev_status, void* ws,
                                    size_t ws_bytes, void* stream);
 
+/* Decode attention without caller workspace (the paper has no counterpart: this is an interface
+ * for callers that cannot allocate device memory, such as a plugin that a host framework hands only
+ * input and output pointers, or a serving loop that must not allocate after start-up).
+ * Same arguments and results as varrate_decode_attn, minus ws/ws_bytes: the scratch lives in a
+ * fixed 4 MiB array in device memory defined by the library (held by every GPU that loads the
+ * library until the process exits). Nothing is allocated, by this call or by the library.
+ *  - Returns VARRATE_ERR_WORKSPACE when the shape needs more than 4 MiB of decode scratch
+ *    (varrate_workspace_bytes(cfg, VARRATE_CALL_DECODE) > 4 MiB).
+ *  - The first call on a device looks up the array's device address (once per device, for the
+ *    current device); make that first call before any stream capture.
+ *  - All calls share the one array: calls that overlap on the GPU (other streams, other host
+ *    threads) race on it and must be serialised by the caller. No contents carry over that matter:
+ *    every scratch element is written before it is read. */
+varrate_status varrate_decode_attn_noalloc(const varrate_config* cfg, const varrate_packed* cache,
+                                           const void* basis_k, const void* basis_v, const void* q,
+                                           int32_t layer, const void* tail_k, const void* tail_v,
+                                           int32_t n_tail, void* out, int32_t* dev_status,
+                                           void* stream);
+
 #ifdef __cplusplus
 }
 #endif

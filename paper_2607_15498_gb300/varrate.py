@@ -65,6 +65,11 @@ _SIGS = {
                                              _c_void_p, ctypes.c_int32, _c_void_p, _c_void_p,
                                              ctypes.c_int32, _c_void_p, _c_void_p, _c_void_p,
                                              ctypes.c_size_t, _c_void_p]),
+    "varrate_decode_attn_noalloc": (ctypes.c_int32, [ctypes.POINTER(varrate_config),
+                                                     ctypes.POINTER(varrate_packed), _c_void_p,
+                                                     _c_void_p, _c_void_p, ctypes.c_int32,
+                                                     _c_void_p, _c_void_p, ctypes.c_int32,
+                                                     _c_void_p, _c_void_p, _c_void_p]),
 }
 
 EXPORTED = tuple(_SIGS)
@@ -178,6 +183,14 @@ def varrate_decode_attn(cfg, packed, basis_k, basis_v, q, layer, tail_k, tail_v,
                                      _ptr(basis_v), _ptr(q), layer, _ptr(tail_k), _ptr(tail_v),
                                      n_tail, _ptr(out), _ptr(dev_status), _ptr(ws), _nbytes(ws),
                                      _stream(stream))
+
+
+def varrate_decode_attn_noalloc(cfg, packed, basis_k, basis_v, q, layer, tail_k, tail_v, n_tail,
+                                out, dev_status, stream=None) -> int:
+    return lib().varrate_decode_attn_noalloc(ctypes.byref(cfg), ctypes.byref(packed.c),
+                                             _ptr(basis_k), _ptr(basis_v), _ptr(q), layer,
+                                             _ptr(tail_k), _ptr(tail_v), n_tail, _ptr(out),
+                                             _ptr(dev_status), _stream(stream))
 
 
 # ------------------------------------------------------------- device-memory plumbing
