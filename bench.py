@@ -322,8 +322,14 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=1)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--layers", type=int, default=None, help="override the layer count (profiling)")
+    ap.add_argument("--batch", type=int, default=None, help="override the sequence count (profiling)")
     args = ap.parse_args()
     wl = synth.workload(args.workload)
+    if args.layers is not None:
+        wl = wl.with_(n_layers=args.layers)
+    if args.batch is not None:
+        wl = wl.with_(batch=args.batch)
     if args.decode_steps is None:
         args.decode_steps = wl.decode_steps
     world, rank, local = dist_env()

@@ -1,0 +1,529 @@
+// Step 4, bf16 — decode attention on the packed coefficients with tensor-core tiles.
+//
+// Same mathematics as decode.cu (attention of Sec. 3.1 over the cache of Eq. 5, never rebuilding K
+// or V): per query head h of KV head g, q~ = U_K q * log2(e)/sqrt(d); score_t = q~[:r_t].c^K_t;
+// o = U_V^T (sum_t 2^(score_t - m) c^V_t) / sum_t 2^(score_t - m).
+//
+// Work split. The coefficient streams of all (sequence, KV head) pairs of the layer form one cost
+// line (element offsets, K stream); the persistent grid (one CTA per SM) cuts it into equal
+// ranges, so every SM moves the same number of bytes. A CTA walks the (sequence, head) segments its
+// range touches; per segment it rotates the query with mma.sync (U_K tile x q), then its warps take
+// 128-slot items of one rank bucket round-robin. An item of rank r is 2 * ceil(r/16) chunks of 16
+// coefficient rows x 128 slots (4 KB): all K chunks, then all V chunks.
+//
+// Memory path. Each warp owns a 4-stage shared-memory ring filled with 16-byte cp.async copies
+// (zero-fill covers rows >= r and slots past the bucket), always 3 chunks ahead of the chunk it
+// computes on, across item boundaries: loads never wait on arithmetic.
+//
+// Arithmetic (per warp, fp32 accumulate, all operands exact or split hi+lo in bf16):
+//   scores   S^T[slot][head] += K^T[slot][j] * Q~^T[j][head]   (mma m16n8k16; K via ldmatrix.trans,
+//            q~ split hi+lo so the product is accurate to ~2^-16)
+//   softmax  online, per head, 8 heads per tile (grp <= 8; unused heads are computed and ignored)
+//   values   O~^T[j][head] += V[j][slot] * P^T[slot][head]      (P split hi+lo, transposed from
+//            the score fragments with movmatrix)
+// Partials (max, sum, o~[128]) per (segment, CTA) go to the workspace; decode_combine_mma merges
+// them, rotates back with U_V^T (staged in shared memory) and normalises.
+#include <stddef.h>
+
+#include "common.cuh"
+#include "kernels.h"
+
+namespace vr {
+
+namespace {
+
+constexpr int kMaxR = kHeadDim;
+constexpr int NW = 8;                 // warps per CTA
+constexpr int ST = 4;                 // ring stages per warp
+constexpr int ISL = 128;              // slots per item
+constexpr int ROWB = ISL * 2 + 16;    // bytes per staged row (+16 B: conflict-free ldmatrix)
+constexpr int STAGE = 16 * ROWB;      // one chunk: 16 rows
+constexpr int kPartStride = kHeadDim + 2;
+constexpr int kHeadsPad = 8;
+
+struct SegSmem {
+  alignas(16) uint32_t qfrag[kHeadDim / 16][32][4];   // per j-chunk, per lane: b0 hi, b1 hi, b0 lo, b1 lo (read as uint4)
+  alignas(16) float qt[kHeadsPad][kHeadDim];          // rotated, scaled queries (fp32)
+  long long base[kMaxR + 2];
+  int cnt[kMaxR + 1];
+};
+static_assert(offsetof(SegSmem, qfrag) % 16 == 0, "qfrag is read with 16-byte loads");
+
+struct Merge {
+  float M[NW][kHeadsPad], L[NW][kHeadsPad];
+  float acc[NW][kHeadsPad][kHeadDim];
+};
+
+// Iterator over this warp's items inside a cost range [lo, hi) of one stream: items are visited
+// in (rank, slot) order and dealt round-robin to the NW warps.
+struct ItemIter {
+  int r;            // current bucket
+  long long it;     // current item index in bucket
+  long long it_end; // end of this bucket's items inside the range
+  int k;            // CTA-local index of item `it`
+};
+
+__device__ __forceinline__ void bucket_range(const SegSmem& sm, int r, long long lo, long long hi,
+                                             long long& i0, long long& i1) {
+  const int n = sm.cnt[r];
+  if (n == 0) { i0 = i1 = 0; return; }
+  const long long n8 = pad8(n), b0 = sm.base[r], unit = (long long)ISL * r;
+  const long long nit = (n8 + ISL - 1) / ISL;
+  i0 = lo > b0 ? (lo - b0 + unit - 1) / unit : 0;
+  i1 = hi > b0 ? (hi - b0 + unit - 1) / unit : 0;
+  if (i1 > nit) i1 = nit;
+  if (i0 > i1) i0 = i1;
+}
+
+// Advance `s` to the next item owned by `warp` (possibly the current one). false when exhausted.
+__device__ __forceinline__ bool iter_seek(ItemIter& s, const SegSmem& sm, long long lo, long long hi,
+                                          int r_max, int warp) {
+  while (true) {
+    while (s.it >= s.it_end) {
+      if (++s.r > r_max) return false;
+      bucket_range(sm, s.r, lo, hi, s.it, s.it_end);
+    }
+    const int skip = ((warp - s.k) % NW + NW) % NW;
+    if (skip == 0) return true;
+    const long long avail = s.it_end - s.it;
+    if (skip < avail) { s.it += skip; s.k += skip; return true; }
+    s.it = s.it_end;
+    s.k += (int)avail;
+  }
+}
+
+__device__ __forceinline__ void iter_step(ItemIter& s) { ++s.it; ++s.k; }
+
+// Producer cursor: which chunk of which item comes next in this warp's stream.
+struct Prod {
+  ItemIter items;
+  bool live;   // items remain
+  int phase;   // 0 = K rows, 1 = V rows
+  int jc;      // 16-row chunk index
+};
+
+__device__ __forceinline__ void issue_chunk(Prod& p, const SegSmem& sm, const __nv_bfloat16* cK,
+                                            const __nv_bfloat16* cV, uint32_t stage_addr,
+                                            long long lo, long long hi, int r_max, int warp,
+                                            int lane) {
+  if (p.live) {
+    const int r = p.items.r;
+    const long long n8 = pad8(sm.cnt[r]);
+    const long long s_begin = p.items.it * ISL;
+    const long long count = min((long long)ISL, n8 - s_begin);
+    const __nv_bfloat16* src0 = (p.phase ? cV : cK) + sm.base[r] + s_begin;
+    const int j0 = p.jc * 16;
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      const int idx = lane + 32 * q;
+      const int row = idx >> 4, col = idx & 15;
+      const int j = j0 + row;
+      const bool ok = (j < r) && (col * 8 < count);
+      const __nv_bfloat16* src = ok ? src0 + (long long)j * n8 + col * 8 : cK;
+      cp_async16(stage_addr + row * ROWB + col * 16, src, ok ? 16u : 0u);
+    }
+    // advance
+    const int nj = (r + 15) >> 4;
+    if (++p.jc == nj) {
+      p.jc = 0;
+      if (++p.phase == 2) {
+        p.phase = 0;
+        iter_step(p.items);
+        p.live = iter_seek(p.items, sm, lo, hi, r_max, warp);
+      }
+    }
+  }
+  cp_async_commit();
+}
+
+// Rotate the queries of (b, g) into the basis: qt[head][j] = scale * sum_i U_K[j][i] q[head][i],
+// warp w computing rows j in [16w, 16w + 16) with one m16n8k16 tile per 16 columns of U_K.
+__device__ void rotate_queries(SegSmem& sm, const __nv_bfloat16* __restrict__ U,
+                               const __nv_bfloat16* __restrict__ q, int grp, int warp, int lane) {
+  const int g8 = lane >> 2, c = lane & 3;
+  const float scale = kLog2e * rsqrtf((float)kHeadDim);
+  for (int mt = warp; mt < kHeadDim / 16; mt += NW) {
+    float d[4] = {0.f, 0.f, 0.f, 0.f};
+    const int j0 = mt * 16;
+#pragma unroll
+    for (int kc = 0; kc < kHeadDim / 16; ++kc) {
+      const int i0 = kc * 16;
+      uint32_t a[4];
+      const uint32_t* Uw = reinterpret_cast<const uint32_t*>(U);
+      a[0] = __ldg(Uw + ((j0 + g8) * kHeadDim + i0 + 2 * c) / 2);
+      a[1] = __ldg(Uw + ((j0 + g8 + 8) * kHeadDim + i0 + 2 * c) / 2);
+      a[2] = __ldg(Uw + ((j0 + g8) * kHeadDim + i0 + 2 * c + 8) / 2);
+      a[3] = __ldg(Uw + ((j0 + g8 + 8) * kHeadDim + i0 + 2 * c + 8) / 2);
+      uint32_t b0 = 0, b1 = 0;
+      if (g8 < grp) {
+        const uint32_t* qw = reinterpret_cast<const uint32_t*>(q + (long long)g8 * kHeadDim);
+        b0 = __ldg(qw + (i0 + 2 * c) / 2);
+        b1 = __ldg(qw + (i0 + 2 * c + 8) / 2);
+      }
+      mma_bf16_16816(d, a, b0, b1);
+    }
+    // d: rows j0+g8 (+8), heads 2c, 2c+1
+    sm.qt[2 * c][j0 + g8] = d[0] * scale;
+    sm.qt[2 * c + 1][j0 + g8] = d[1] * scale;
+    sm.qt[2 * c][j0 + g8 + 8] = d[2] * scale;
+    sm.qt[2 * c + 1][j0 + g8 + 8] = d[3] * scale;
+  }
+}
+
+// Score-MMA B fragments of q~ (split hi + lo) for every 16-row chunk, one uint4 per lane.
+__device__ void build_qfrag(SegSmem& sm, int tid) {
+  for (int i = tid; i < (kHeadDim / 16) * 32; i += NW * 32) {
+    const int jc = i / 32, lane = i % 32, g8 = lane >> 2, c = lane & 3;
+    const int j = jc * 16 + 2 * c;
+    uint32_t h0, l0, h1, l1;
+    split_bf16(sm.qt[g8][j], sm.qt[g8][j + 1], h0, l0);
+    split_bf16(sm.qt[g8][j + 8], sm.qt[g8][j + 9], h1, l1);
+    sm.qfrag[jc][lane][0] = h0;
+    sm.qfrag[jc][lane][1] = h1;
+    sm.qfrag[jc][lane][2] = l0;
+    sm.qfrag[jc][lane][3] = l1;
+  }
+}
+
+__global__ void __launch_bounds__(NW * 32, 1)
+decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restrict__ bucket_count,
+                  const int64_t* __restrict__ bucket_base, const __nv_bfloat16* __restrict__ basis_k,
+                  const __nv_bfloat16* __restrict__ qin, float* __restrict__ part,
+                  int32_t* __restrict__ dev_status, Shape s, int layer) {
+  extern __shared__ __align__(128) unsigned char smem[];
+  unsigned char* ring = smem;                                     // NW * ST * STAGE
+  static_assert((NW * ST * STAGE) % 16 == 0, "SegSmem must start 16-byte aligned");
+  SegSmem& sm = *reinterpret_cast<SegSmem*>(smem + NW * ST * STAGE);
+  Merge& mg = *reinterpret_cast<Merge*>(smem);                    // aliases the ring
+  __shared__ long long segW[64];                                  // per-sequence stream length
+
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int g8 = lane >> 2, c = lane & 3;
+  const int C = gridDim.x, cta = blockIdx.x;
+
+  // stream length of every sequence of this layer (same for every head); poisoned tables -> 0
+  for (int b = tid; b < s.B; b += blockDim.x) {
+    const long long w = bucket_base[((long long)b * s.L + layer) * (kMaxR + 2) + kMaxR + 1];
+    segW[b] = (w >= 0 && w <= s.cap) ? w : 0;
+  }
+  // the ring only ever holds finite coefficients or zeros
+  for (int i = tid; i < NW * ST * STAGE / 16; i += blockDim.x)
+    reinterpret_cast<uint4*>(ring)[i] = make_uint4(0, 0, 0, 0);
+  __syncthreads();
+  long long T = 0;
+  for (int b = 0; b < s.B; ++b) T += segW[b] * s.G;
+  if (T == 0) return;
+  const long long lo_g = (long long)((__int128)T * cta / C);
+  const long long hi_g = (long long)((__int128)T * (cta + 1) / C);
+
+  long long P = 0;   // start of segment (b, g) on the cost line
+  for (int b = 0; b < s.B; ++b) {
+    const long long W = segW[b];
+    for (int g = 0; g < s.G; ++g, P += W) {
+      if (W == 0 || P + W <= lo_g || P >= hi_g) continue;
+      const long long lo = max(lo_g, P) - P, hi = min(hi_g, P + W) - P;
+      const long long bl = (long long)b * s.L + layer;
+      __syncthreads();
+      for (int r = tid; r <= kMaxR + 1; r += blockDim.x) {
+        if (r <= kMaxR) sm.cnt[r] = bucket_count[bl * (kMaxR + 1) + r];
+        sm.base[r] = bucket_base[bl * (kMaxR + 2) + r];
+      }
+      rotate_queries(sm, basis_k + ((long long)layer * s.G + g) * kHeadDim * kHeadDim,
+                     qin + ((long long)b * s.H + (long long)g * s.grp) * kHeadDim, s.grp, warp, lane);
+      __syncthreads();
+      build_qfrag(sm, tid);
+      __syncthreads();
+
+      const __nv_bfloat16* cK = coef + ((bl * s.G + g) * 2) * s.cap;
+      const __nv_bfloat16* cV = cK + s.cap;
+      const uint32_t ring_w = smem_addr(ring) + warp * ST * STAGE;
+
+      float Mx[2] = {-INFINITY, -INFINITY}, Ls[2] = {0.f, 0.f};
+      float oacc[kHeadDim / 16][4];
+#pragma unroll
+      for (int t = 0; t < kHeadDim / 16; ++t) oacc[t][0] = oacc[t][1] = oacc[t][2] = oacc[t][3] = 0.f;
+
+      Prod pr;
+      pr.items.r = s.r_min - 1; pr.items.it = pr.items.it_end = 0; pr.items.k = 0;
+      pr.live = iter_seek(pr.items, sm, lo, hi, s.r_max, warp);
+      pr.phase = 0; pr.jc = 0;
+      ItemIter cons = pr.items;
+      bool cons_live = pr.live;
+      int stage_p = 0, stage_c = 0;
+#pragma unroll
+      for (int i = 0; i < ST - 1; ++i) {
+        issue_chunk(pr, sm, cK, cV, ring_w + stage_p * STAGE, lo, hi, s.r_max, warp, lane);
+        stage_p = (stage_p + 1) % ST;
+      }
+
+      while (cons_live) {
+        const int r = cons.r;
+        const int nj = (r + 15) >> 4;
+        const long long n_real = sm.cnt[r] - cons.it * ISL;   // real slots of this item (may exceed ISL)
+        float sc[ISL / 16][4];
+#pragma unroll
+        for (int t = 0; t < ISL / 16; ++t) sc[t][0] = sc[t][1] = sc[t][2] = sc[t][3] = 0.f;
+
+        // ---- K chunks: scores
+        for (int jc = 0; jc < nj; ++jc) {
+          cp_async_wait<ST - 2>();
+          __syncwarp();
+          const uint32_t st_addr = ring_w + stage_c * STAGE;
+          const uint4 qf = *reinterpret_cast<const uint4*>(&sm.qfrag[jc][lane][0]);
+          const int m = lane >> 3, r8 = lane & 7;
+          const uint32_t a_base = st_addr + ((m >> 1) * 8 + r8) * ROWB + (m & 1) * 16;
+#pragma unroll
+          for (int mt = 0; mt < ISL / 16; ++mt) {
+            uint32_t a[4];
+            ldsm_x4_trans(a_base + mt * 32, a);
+            mma_bf16_16816(sc[mt], a, qf.x, qf.y);
+            mma_bf16_16816(sc[mt], a, qf.z, qf.w);
+          }
+          __syncwarp();
+          issue_chunk(pr, sm, cK, cV, ring_w + stage_p * STAGE, lo, hi, s.r_max, warp, lane);
+          stage_p = (stage_p + 1) % ST;
+          stage_c = (stage_c + 1) % ST;
+        }
+
+        // ---- online softmax over the item's slots (heads 2c, 2c+1 per lane)
+        float mloc[2] = {-INFINITY, -INFINITY};
+#pragma unroll
+        for (int mt = 0; mt < ISL / 16; ++mt) {
+          const int s0 = mt * 16 + g8;
+          if (s0 >= n_real) { sc[mt][0] = sc[mt][1] = -INFINITY; }
+          if (s0 + 8 >= n_real) { sc[mt][2] = sc[mt][3] = -INFINITY; }
+          mloc[0] = fmaxf(mloc[0], fmaxf(sc[mt][0], sc[mt][2]));
+          mloc[1] = fmaxf(mloc[1], fmaxf(sc[mt][1], sc[mt][3]));
+        }
+#pragma unroll
+        for (int o = 4; o < 32; o <<= 1) {
+          mloc[0] = fmaxf(mloc[0], __shfl_xor_sync(0xffffffffu, mloc[0], o));
+          mloc[1] = fmaxf(mloc[1], __shfl_xor_sync(0xffffffffu, mloc[1], o));
+        }
+        float corr[2];
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+          const float nm = fmaxf(Mx[e], mloc[e]);
+          corr[e] = fast_exp2(Mx[e] - nm);
+          Mx[e] = nm;
+        }
+        float lsum[2] = {0.f, 0.f};
+        uint32_t pb[ISL / 16][4];   // per slot tile: b0 hi, b1 hi, b0 lo, b1 lo
+#pragma unroll
+        for (int mt = 0; mt < ISL / 16; ++mt) {
+          const float p0 = fast_exp2(sc[mt][0] - Mx[0]), p1 = fast_exp2(sc[mt][1] - Mx[1]);
+          const float p2 = fast_exp2(sc[mt][2] - Mx[0]), p3 = fast_exp2(sc[mt][3] - Mx[1]);
+          lsum[0] += p0 + p2;
+          lsum[1] += p1 + p3;
+          uint32_t h01, l01, h23, l23;
+          split_bf16(p0, p1, h01, l01);
+          split_bf16(p2, p3, h23, l23);
+          pb[mt][0] = movmatrix_trans(h01);
+          pb[mt][1] = movmatrix_trans(h23);
+          pb[mt][2] = movmatrix_trans(l01);
+          pb[mt][3] = movmatrix_trans(l23);
+        }
+        Ls[0] = Ls[0] * corr[0] + lsum[0];
+        Ls[1] = Ls[1] * corr[1] + lsum[1];
+#pragma unroll
+        for (int t = 0; t < kHeadDim / 16; ++t) {
+          oacc[t][0] *= corr[0]; oacc[t][1] *= corr[1];
+          oacc[t][2] *= corr[0]; oacc[t][3] *= corr[1];
+        }
+
+        // ---- V chunks: weighted coefficient rows
+#pragma unroll
+        for (int jc = 0; jc < kHeadDim / 16; ++jc) {
+          if (jc >= nj) break;
+          cp_async_wait<ST - 2>();
+          __syncwarp();
+          const uint32_t st_addr = ring_w + stage_c * STAGE;
+          const int m = lane >> 3, r8 = lane & 7;
+          const uint32_t a_base = st_addr + ((m & 1) * 8 + r8) * ROWB + (m >> 1) * 16;
+#pragma unroll
+          for (int kt = 0; kt < ISL / 16; ++kt) {
+            uint32_t a[4];
+            ldsm_x4(a_base + kt * 32, a);
+            mma_bf16_16816(oacc[jc], a, pb[kt][0], pb[kt][1]);
+            mma_bf16_16816(oacc[jc], a, pb[kt][2], pb[kt][3]);
+          }
+          __syncwarp();
+          issue_chunk(pr, sm, cK, cV, ring_w + stage_p * STAGE, lo, hi, s.r_max, warp, lane);
+          stage_p = (stage_p + 1) % ST;
+          stage_c = (stage_c + 1) % ST;
+        }
+        iter_step(cons);
+        cons_live = iter_seek(cons, sm, lo, hi, s.r_max, warp);
+      }
+      cp_async_wait<0>();
+
+      // ---- merge the warps of this CTA for this segment
+#pragma unroll
+      for (int e = 0; e < 2; ++e)
+#pragma unroll
+        for (int o = 4; o < 32; o <<= 1) Ls[e] += __shfl_xor_sync(0xffffffffu, Ls[e], o);
+      __syncthreads();   // every warp is done with its ring
+      if (g8 == 0) {
+        mg.M[warp][2 * c] = Mx[0]; mg.M[warp][2 * c + 1] = Mx[1];
+        mg.L[warp][2 * c] = Ls[0]; mg.L[warp][2 * c + 1] = Ls[1];
+      }
+#pragma unroll
+      for (int t = 0; t < kHeadDim / 16; ++t) {
+        mg.acc[warp][2 * c][t * 16 + g8] = oacc[t][0];
+        mg.acc[warp][2 * c + 1][t * 16 + g8] = oacc[t][1];
+        mg.acc[warp][2 * c][t * 16 + g8 + 8] = oacc[t][2];
+        mg.acc[warp][2 * c + 1][t * 16 + g8 + 8] = oacc[t][3];
+      }
+      __syncthreads();
+      // partial slot of this (segment, CTA): index cta + segment number (unique, see combine)
+      const long long seg = (long long)b * s.G + g;
+      float* out = part + (cta + seg) * (long long)kHeadsPad * kPartStride;
+      for (int i = tid; i < kHeadsPad * kHeadDim; i += blockDim.x) {
+        const int h = i / kHeadDim, j = i % kHeadDim;
+        float mx = -INFINITY;
+#pragma unroll
+        for (int w = 0; w < NW; ++w) mx = fmaxf(mx, mg.M[w][h]);
+        float o = 0.f, l = 0.f;
+        if (mx != -INFINITY) {
+#pragma unroll
+          for (int w = 0; w < NW; ++w) {
+            const float f = fast_exp2(mg.M[w][h] - mx);
+            o = fmaf(mg.acc[w][h][j], f, o);
+            l = fmaf(mg.L[w][h], f, l);
+          }
+        }
+        out[h * kPartStride + j] = o;
+        if (j == 0) { out[h * kPartStride + kHeadDim] = mx; out[h * kPartStride + kHeadDim + 1] = l; }
+      }
+      __syncthreads();   // merge buffers alias the ring of the next segment
+      (void)dev_status;
+    }
+  }
+}
+
+// grid (G, B), 256 threads: merge the partials of segment (b, g), add the exact tail, rotate back.
+__global__ void __launch_bounds__(256)
+decode_combine_mma_kernel(const float* __restrict__ part, const int64_t* __restrict__ bucket_base,
+                          const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __restrict__ basis_v,
+                          const __nv_bfloat16* __restrict__ tail_k, const __nv_bfloat16* __restrict__ tail_v,
+                          int n_tail, __nv_bfloat16* __restrict__ out, Shape s, int layer, int C) {
+  __shared__ __align__(16) __nv_bfloat16 us[kHeadDim * kHeadDim];   // U_V[g], row j
+  __shared__ float ot[kHeadsPad][kHeadDim];
+  __shared__ float qrow[kHeadsPad][kHeadDim];
+  __shared__ float tsc[kHeadsPad][64];
+  __shared__ float hm[kHeadsPad], hl[kHeadsPad];
+  __shared__ long long segW[64];
+  const int g = blockIdx.x, b = blockIdx.y;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+
+  const uint4* src = reinterpret_cast<const uint4*>(basis_v + ((long long)layer * s.G + g) * kHeadDim * kHeadDim);
+  for (int i = tid; i < kHeadDim * kHeadDim / 8; i += blockDim.x) reinterpret_cast<uint4*>(us)[i] = src[i];
+  for (int bb = tid; bb < s.B; bb += blockDim.x) {
+    const long long w = bucket_base[((long long)bb * s.L + layer) * (kMaxR + 2) + kMaxR + 1];
+    segW[bb] = (w >= 0 && w <= s.cap) ? w : 0;
+  }
+  for (int i = tid; i < s.grp * kHeadDim; i += blockDim.x)
+    qrow[i / kHeadDim][i % kHeadDim] =
+        __bfloat162float(q[((long long)b * s.H + (long long)g * s.grp) * kHeadDim + i]);
+  __syncthreads();
+  long long T = 0, P = 0;
+  for (int bb = 0; bb < s.B; ++bb) T += segW[bb] * s.G;
+  for (int bb = 0; bb < b; ++bb) P += segW[bb] * s.G;
+  const long long W = segW[b];
+  P += (long long)g * W;
+  const long long seg = (long long)b * s.G + g;
+  // CTAs whose range [T c / C, T (c+1) / C) meets [P, P + W)
+  int c0 = 0, c1 = -1;
+  if (W > 0 && T > 0) {
+    c0 = (int)((__int128)P * C / T);
+    while (c0 > 0 && (long long)((__int128)T * c0 / C) > P) --c0;
+    while ((long long)((__int128)T * (c0 + 1) / C) <= P) ++c0;
+    c1 = (int)((__int128)(P + W - 1) * C / T);
+    while (c1 + 1 < C && (long long)((__int128)T * (c1 + 1) / C) <= P + W - 1) ++c1;
+    while (c1 > c0 && (long long)((__int128)T * c1 / C) > P + W - 1) --c1;
+  }
+  const float scale = kLog2e * rsqrtf((float)kHeadDim);
+  // per head: global max over partials and tail, then weights
+  if (tid < s.grp) {
+    float mx = -INFINITY;
+    for (int cc = c0; cc <= c1; ++cc) mx = fmaxf(mx, part[((cc + seg) * kHeadsPad + tid) * kPartStride + kHeadDim]);
+    hm[tid] = mx;
+  }
+  // exact tail scores (n_tail <= 64 handled here; larger tails use decode.cu's path)
+  for (int i = warp; i < s.grp * n_tail; i += blockDim.x / 32) {
+    const int h = i / n_tail, t = i % n_tail;
+    const __nv_bfloat16* tk = tail_k + (((long long)b * s.G + g) * n_tail + t) * kHeadDim;
+    float a = 0.f;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) a = fmaf(qrow[h][lane * 4 + k], __bfloat162float(tk[lane * 4 + k]), a);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) a += __shfl_xor_sync(0xffffffffu, a, o);
+    if (lane == 0) tsc[h][t] = a * scale;
+  }
+  __syncthreads();
+  if (tid < s.grp) {
+    float mx = hm[tid];
+    for (int t = 0; t < n_tail; ++t) mx = fmaxf(mx, tsc[tid][t]);
+    float l = 0.f;
+    for (int cc = c0; cc <= c1; ++cc) {
+      const float* pp = part + ((cc + seg) * kHeadsPad + tid) * kPartStride;
+      if (pp[kHeadDim] != -INFINITY) l = fmaf(pp[kHeadDim + 1], exp2f(pp[kHeadDim] - mx), l);
+    }
+    for (int t = 0; t < n_tail; ++t) {
+      tsc[tid][t] = exp2f(tsc[tid][t] - mx);
+      l += tsc[tid][t];
+    }
+    hm[tid] = mx;
+    hl[tid] = l;
+  }
+  __syncthreads();
+  for (int i = tid; i < s.grp * kHeadDim; i += blockDim.x) {
+    const int h = i / kHeadDim, j = i % kHeadDim;
+    float o = 0.f;
+    for (int cc = c0; cc <= c1; ++cc) {
+      const float* pp = part + ((cc + seg) * kHeadsPad + h) * kPartStride;
+      if (pp[kHeadDim] != -INFINITY) o = fmaf(pp[j], exp2f(pp[kHeadDim] - hm[h]), o);
+    }
+    ot[h][j] = o;
+  }
+  __syncthreads();
+  for (int i = tid; i < s.grp * kHeadDim; i += blockDim.x) {
+    const int h = i / kHeadDim, col = i % kHeadDim;
+    float y = 0.f;
+#pragma unroll 8
+    for (int j = 0; j < kHeadDim; ++j) y = fmaf(__bfloat162float(us[j * kHeadDim + col]), ot[h][j], y);
+    for (int t = 0; t < n_tail; ++t)
+      y = fmaf(tsc[h][t], __bfloat162float(tail_v[(((long long)b * s.G + g) * n_tail + t) * kHeadDim + col]), y);
+    out[((long long)b * s.H + (long long)g * s.grp + h) * kHeadDim + col] = __float2bfloat16_rn(y / hl[h]);
+  }
+}
+
+}  // namespace
+
+size_t decode_mma_smem_bytes() { return (size_t)NW * ST * STAGE + sizeof(SegSmem); }
+
+size_t decode_mma_part_bytes(const Shape& s, int num_sms) {
+  return (size_t)(num_sms + (size_t)s.B * s.G) * kHeadsPad * kPartStride * sizeof(float);
+}
+
+bool decode_mma_supported(const Shape& s, int n_tail) {
+  return s.dtype == VARRATE_BF16 && s.B <= 64 && n_tail <= 64 && sizeof(Merge) <= (size_t)NW * ST * STAGE;
+}
+
+int launch_decode_mma(const Shape& s, const varrate_packed& c, const void* basis_k,
+                      const void* basis_v, const void* q, int layer, const void* tail_k,
+                      const void* tail_v, int n_tail, void* out, int32_t* dev_status, float* part,
+                      int num_sms, cudaStream_t st) {
+  const size_t smem = decode_mma_smem_bytes();
+  cudaFuncSetAttribute(decode_mma_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  decode_mma_kernel<<<num_sms, NW * 32, smem, st>>>(
+      (const __nv_bfloat16*)c.coef, c.bucket_count, c.bucket_base, (const __nv_bfloat16*)basis_k,
+      (const __nv_bfloat16*)q, part, dev_status, s, layer);
+  decode_combine_mma_kernel<<<dim3(s.G, s.B), 256, 0, st>>>(
+      part, c.bucket_base, (const __nv_bfloat16*)q, (const __nv_bfloat16*)basis_v,
+      (const __nv_bfloat16*)tail_k, (const __nv_bfloat16*)tail_v, n_tail, (__nv_bfloat16*)out, s,
+      layer, num_sms);
+  return 2;
+}
+
+}  // namespace vr

@@ -32,9 +32,23 @@ int launch_pack(const Shape& s, const void* k, const void* v, const void* basis_
                 const void* basis_v, const varrate_packed& out, int32_t* dev_status,
                 int num_sms, cudaStream_t st);
 
+// bf16 tensor-core projection (project_tc.cu)
+size_t project_tc_smem_bytes();
+int launch_project_tc(const Shape& s, const void* k, const void* v, const void* basis_k,
+                      const void* basis_v, const varrate_packed& out, int32_t* dev_status,
+                      int num_sms, cudaStream_t st);
+
 // ---- step 4: decode attention
 int decode_splits(const Shape& s, int num_sms);
 size_t decode_ws_bytes(const Shape& s, int num_sms);
+// bf16 tensor-core decode (decode_mma.cu)
+size_t decode_mma_smem_bytes();
+size_t decode_mma_part_bytes(const Shape& s, int num_sms);
+bool decode_mma_supported(const Shape& s, int n_tail);
+int launch_decode_mma(const Shape& s, const varrate_packed& c, const void* basis_k,
+                      const void* basis_v, const void* q, int layer, const void* tail_k,
+                      const void* tail_v, int n_tail, void* out, int32_t* dev_status, float* part,
+                      int num_sms, cudaStream_t st);
 int launch_decode(const Shape& s, const varrate_packed& cache, const void* basis_k,
                   const void* basis_v, const void* q, int layer, const void* tail_k,
                   const void* tail_v, int n_tail, void* out, int32_t* dev_status, void* ws,

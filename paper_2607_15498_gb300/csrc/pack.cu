@@ -226,10 +226,7 @@ int launch_pack(const Shape& s, const void* k, const void* v, const void* basis_
     using T = __nv_bfloat16;
     pack_tables_kernel<T><<<s.B * s.L, 1024, 0, st>>>(out.ranks, out.bucket_count, out.bucket_base,
                                                       out.perm, out.pos, (T*)out.coef, dev_status, s);
-    cudaFuncSetAttribute(project_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    project_kernel<T><<<grid, 256, smem, st>>>((const T*)k, (const T*)v, (const T*)basis_k,
-                                               (const T*)basis_v, out.ranks, out.bucket_count,
-                                               out.bucket_base, out.perm, out.pos, (T*)out.coef, s, chunk);
+    return 1 + launch_project_tc(s, k, v, basis_k, basis_v, out, dev_status, num_sms, st);
   } else {
     using T = float;
     pack_tables_kernel<T><<<s.B * s.L, 1024, 0, st>>>(out.ranks, out.bucket_count, out.bucket_base,
