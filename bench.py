@@ -296,6 +296,20 @@ def run_oracle_sample(wl, budget_s: float = 15.0, decode_steps: int = 2, seed_la
             "steps": n, "input_s": t_in}
 
 
+def reduce_over_ranks(total_s, dec_s, enc_ms_per_ctx, world, device):
+    """Max of each timing over all ranks (the job is as slow as its slowest rank)."""
+    if world <= 1:
+        return total_s, dec_s, enc_ms_per_ctx
+    t = torch.tensor([total_s, dec_s, enc_ms_per_ctx], dtype=torch.float64, device=device)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return tuple(t.tolist())
+
+
+def job_decode_gbs(world, steps, step_dec_bytes, dec_s):
+    """Whole-job decode throughput: bytes every rank moved over the slowest rank's time."""
+    return world * steps * step_dec_bytes / dec_s / 1e9
+
+
 def cpu_cores():
     try:
         return len(os.sched_getaffinity(0))
@@ -378,11 +392,8 @@ def main():
     total_s = r["total_ms"] * 1e-3
     dec_s = sum(r["dec_ms"]) * 1e-3
     enc_ms_per_ctx = statistics.mean(r["enc_ms"]) / wl.batch
-    if world > 1:
-        t = torch.tensor([total_s, dec_s, enc_ms_per_ctx], dtype=torch.float64, device="cuda")
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        total_s, dec_s, enc_ms_per_ctx = t.tolist()
-    dec_gbs = world * K * r["step_dec_bytes"] / dec_s / 1e9
+    total_s, dec_s, enc_ms_per_ctx = reduce_over_ranks(total_s, dec_s, enc_ms_per_ctx, world, "cuda")
+    dec_gbs = job_decode_gbs(world, K, r["step_dec_bytes"], dec_s)
     calls = [c for step in r["call_ms"] for c in step]
     avg_call_ms = statistics.mean(calls)
     bytes_per_call = statistics.mean(r["dec_bytes"])

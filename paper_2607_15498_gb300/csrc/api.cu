@@ -135,7 +135,8 @@ varrate_status varrate_salience(const varrate_config* cfg, const void* q_win, co
   const size_t need = ws_bytes(cfg, VARRATE_CALL_SALIENCE);
   if (ws_bytes_ < need || (need > 0 && ws == nullptr)) return VARRATE_ERR_WORKSPACE;
   const Shape s = make_shape(cfg, cap_elems(cfg));
-  vr::launch_salience(s, q_win, k, sal_out, ws, num_sms(), (cudaStream_t)stream);
+  if (vr::launch_salience(s, q_win, k, sal_out, ws, nullptr, num_sms(), (cudaStream_t)stream) < 0)
+    return VARRATE_ERR_CUDA;
   return launched();
 }
 
@@ -181,7 +182,8 @@ varrate_status varrate_encode(const varrate_config* cfg, const void* q_win, cons
   int64_t* realized = realized_sum
       ? realized_sum
       : reinterpret_cast<int64_t*>(w + sal_ws + align256((size_t)s.B * s.L * s.n_coded * sizeof(float)));
-  if (cfg->mode == VARRATE_SALIENCE) vr::launch_salience(s, q_win, k, sal, w, sms, cs);
+  if (cfg->mode == VARRATE_SALIENCE && vr::launch_salience(s, q_win, k, sal, w, dev_status, sms, cs) < 0)
+    return VARRATE_ERR_CUDA;
   vr::launch_allocate(s, sal, out->ranks, realized, dev_status, cs);
   vr::launch_pack(s, k, v, basis_k, basis_v, *out, dev_status, sms, cs);
   return launched();

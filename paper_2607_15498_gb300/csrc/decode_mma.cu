@@ -8,19 +8,20 @@
 // line (element offsets, K stream); the persistent grid (one CTA per SM) cuts it into equal
 // ranges, so every SM moves the same number of bytes. A CTA walks the (sequence, head) segments its
 // range touches; per segment it rotates the query with mma.sync (U_K tile x q), then its warps take
-// 128-slot items of one rank bucket round-robin. An item of rank r is 2 * ceil(r/16) chunks of 16
-// coefficient rows x 128 slots (4 KB): all K chunks, then all V chunks.
+// 128-slot items of one rank bucket round-robin. An item of rank r is 2 * ceil(r/32) chunks of 32
+// coefficient rows x 128 slots (8 KB): all K chunks, then all V chunks.
 //
-// Memory path. Each warp owns a 4-stage shared-memory ring filled with 16-byte cp.async copies
-// (zero-fill covers rows >= r and slots past the bucket), always 3 chunks ahead of the chunk it
-// computes on, across item boundaries: loads never wait on arithmetic.
+// Memory path. Each warp owns a 3-stage shared-memory ring filled by 1-D TMA bulk copies (one per
+// coefficient row, one lane per row) that complete on a per-stage mbarrier; the warp stays 2 chunks
+// ahead of the chunk it computes on, across item boundaries, so loads never wait on arithmetic. Rows >= r of a chunk are never loaded; they are masked out of the tensor-core
+// fragments instead, and the ring only ever holds finite coefficients.
 //
 // Arithmetic (per warp, fp32 accumulate, all operands exact or split hi+lo in bf16):
 //   scores   S^T[slot][head] += K^T[slot][j] * Q~^T[j][head]   (mma m16n8k16; K via ldmatrix.trans,
 //            q~ split hi+lo so the product is accurate to ~2^-16)
 //   softmax  online, per head, 8 heads per tile (grp <= 8; unused heads are computed and ignored)
-//   values   O~^T[j][head] += V[j][slot] * P^T[slot][head]      (P split hi+lo, transposed from
-//            the score fragments with movmatrix)
+//   values   O~^T[j][head] += V[j][slot] * P^T[slot][head]      (P in bf16, <= 2^-9 relative per
+//            weight, transposed from the score fragments with movmatrix)
 // Partials (max, sum, o~[128]) per (segment, CTA) go to the workspace; decode_combine_mma merges
 // them, rotates back with U_V^T (staged in shared memory) and normalises.
 #include <stddef.h>
@@ -34,18 +35,23 @@ namespace {
 
 constexpr int kMaxR = kHeadDim;
 constexpr int NW = 8;                 // warps per CTA
-constexpr int ST = 4;                 // ring stages per warp
+constexpr int ST = 3;                 // ring stages per warp
 constexpr int ISL = 128;              // slots per item
+constexpr int CH = 32;                // coefficient rows per chunk
 constexpr int ROWB = ISL * 2 + 16;    // bytes per staged row (+16 B: conflict-free ldmatrix)
-constexpr int STAGE = 16 * ROWB;      // one chunk: 16 rows
+constexpr int STAGE = CH * ROWB;      // one chunk: 32 rows
 constexpr int kPartStride = kHeadDim + 2;
 constexpr int kHeadsPad = 8;
+constexpr uint32_t kWaitTries = 1u << 22;   // bounded mbarrier polls (well over a second)
+constexpr float kSlack = 8.f;                // headroom of the running max, log2 units
 
 struct SegSmem {
   alignas(16) uint32_t qfrag[kHeadDim / 16][32][4];   // per j-chunk, per lane: b0 hi, b1 hi, b0 lo, b1 lo (read as uint4)
   alignas(16) float qt[kHeadsPad][kHeadDim];          // rotated, scaled queries (fp32)
   long long base[kMaxR + 2];
   int cnt[kMaxR + 1];
+  int it_lo[kMaxR + 1];     // first item of bucket r inside this CTA's cost range
+  int it_pref[kMaxR + 2];   // exclusive prefix of the per-bucket item counts
 };
 static_assert(offsetof(SegSmem, qfrag) % 16 == 0, "qfrag is read with 16-byte loads");
 
@@ -54,15 +60,9 @@ struct Merge {
   float acc[NW][kHeadsPad][kHeadDim];
 };
 
-// Iterator over this warp's items inside a cost range [lo, hi) of one stream: items are visited
-// in (rank, slot) order and dealt round-robin to the NW warps.
-struct ItemIter {
-  int r;            // current bucket
-  long long it;     // current item index in bucket
-  long long it_end; // end of this bucket's items inside the range
-  int k;            // CTA-local index of item `it`
-};
-
+// Items of one CTA inside its cost range [lo, hi) of a stream, in (rank, slot) order: item k lies
+// in bucket r with it_pref[r] <= k < it_pref[r + 1] and is item it_lo[r] + (k - it_pref[r]) of that
+// bucket. Warp w takes items w, w + NW, w + 2 NW, ...
 __device__ __forceinline__ void bucket_range(const SegSmem& sm, int r, long long lo, long long hi,
                                              long long& i0, long long& i1) {
   const int n = sm.cnt[r];
@@ -75,65 +75,66 @@ __device__ __forceinline__ void bucket_range(const SegSmem& sm, int r, long long
   if (i0 > i1) i0 = i1;
 }
 
-// Advance `s` to the next item owned by `warp` (possibly the current one). false when exhausted.
-__device__ __forceinline__ bool iter_seek(ItemIter& s, const SegSmem& sm, long long lo, long long hi,
-                                          int r_max, int warp) {
-  while (true) {
-    while (s.it >= s.it_end) {
-      if (++s.r > r_max) return false;
-      bucket_range(sm, s.r, lo, hi, s.it, s.it_end);
-    }
-    const int skip = ((warp - s.k) % NW + NW) % NW;
-    if (skip == 0) return true;
-    const long long avail = s.it_end - s.it;
-    if (skip < avail) { s.it += skip; s.k += skip; return true; }
-    s.it = s.it_end;
-    s.k += (int)avail;
-  }
-}
+struct Item {
+  int r;    // bucket (rank)
+  int it;   // item index inside the bucket
+};
 
-__device__ __forceinline__ void iter_step(ItemIter& s) { ++s.it; ++s.k; }
+__device__ __forceinline__ Item item_at(const SegSmem& sm, int k) {
+  int lo = 0, hi = kMaxR + 1;   // it_pref[lo] <= k < it_pref[hi]
+  while (hi - lo > 1) {
+    const int mid = (lo + hi) >> 1;
+    if (sm.it_pref[mid] <= k) lo = mid; else hi = mid;
+  }
+  Item x;
+  x.r = lo;
+  x.it = sm.it_lo[lo] + (k - sm.it_pref[lo]);
+  return x;
+}
 
 // Producer cursor: which chunk of which item comes next in this warp's stream.
 struct Prod {
-  ItemIter items;
-  bool live;   // items remain
+  int k;       // item index (CTA-local)
+  Item item;
   int phase;   // 0 = K rows, 1 = V rows
   int jc;      // 16-row chunk index
 };
 
-__device__ __forceinline__ void issue_chunk(Prod& p, const SegSmem& sm, const __nv_bfloat16* cK,
+// Issue the next chunk of this warp's stream into `stage` (one lane per row).
+// Returns false (and issues nothing) when the stream is exhausted.
+__device__ __forceinline__ bool issue_chunk(Prod& p, const SegSmem& sm, const __nv_bfloat16* cK,
                                             const __nv_bfloat16* cV, uint32_t stage_addr,
-                                            long long lo, long long hi, int r_max, int warp,
-                                            int lane) {
-  if (p.live) {
-    const int r = p.items.r;
-    const long long n8 = pad8(sm.cnt[r]);
-    const long long s_begin = p.items.it * ISL;
-    const long long count = min((long long)ISL, n8 - s_begin);
-    const __nv_bfloat16* src0 = (p.phase ? cV : cK) + sm.base[r] + s_begin;
-    const int j0 = p.jc * 16;
-#pragma unroll
-    for (int q = 0; q < 8; ++q) {
-      const int idx = lane + 32 * q;
-      const int row = idx >> 4, col = idx & 15;
-      const int j = j0 + row;
-      const bool ok = (j < r) && (col * 8 < count);
-      const __nv_bfloat16* src = ok ? src0 + (long long)j * n8 + col * 8 : cK;
-      cp_async16(stage_addr + row * ROWB + col * 16, src, ok ? 16u : 0u);
-    }
-    // advance
-    const int nj = (r + 15) >> 4;
-    if (++p.jc == nj) {
-      p.jc = 0;
-      if (++p.phase == 2) {
-        p.phase = 0;
-        iter_step(p.items);
-        p.live = iter_seek(p.items, sm, lo, hi, r_max, warp);
-      }
+                                            uint64_t* bar, int total, int lane) {
+  if (p.k >= total) return false;
+  const int r = p.item.r;
+  const long long n8 = pad8(sm.cnt[r]);
+  const long long s_begin = (long long)p.item.it * ISL;
+  const uint32_t row_bytes = (uint32_t)min((long long)ISL, n8 - s_begin) * 2u;   // multiple of 16
+  const int j0 = p.jc * CH;
+  const int rows = min(CH, r - j0);
+  if (lane == 0) mbar_arrive_expect_tx(bar, row_bytes * (uint32_t)rows);
+  __syncwarp();
+  fence_proxy_async_smem();   // earlier ldmatrix reads of this stage precede the async writes
+  if (lane < rows) {
+    const __nv_bfloat16* src = (p.phase ? cV : cK) + sm.base[r] + (long long)(j0 + lane) * n8 + s_begin;
+    bulk_g2s(stage_addr + lane * ROWB, src, row_bytes, bar);
+  }
+  const int nj = (r + CH - 1) / CH;
+  if (++p.jc == nj) {
+    p.jc = 0;
+    if (++p.phase == 2) {
+      p.phase = 0;
+      p.k += NW;
+      if (p.k < total) p.item = item_at(sm, p.k);
     }
   }
-  cp_async_commit();
+  return true;
+}
+
+// Keep the bf16 halves of `w` whose row index (lo half: j, hi half: j + 1) is below r.
+__device__ __forceinline__ uint32_t keep_rows(uint32_t w, int j, int r) {
+  const uint32_t m = (j < r ? 0x0000FFFFu : 0u) | (j + 1 < r ? 0xFFFF0000u : 0u);
+  return w & m;
 }
 
 // Rotate the queries of (b, g) into the basis: qt[head][j] = scale * sum_i U_K[j][i] q[head][i],
@@ -194,25 +195,37 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
   unsigned char* ring = smem;                                     // NW * ST * STAGE
   static_assert((NW * ST * STAGE) % 16 == 0, "SegSmem must start 16-byte aligned");
   SegSmem& sm = *reinterpret_cast<SegSmem*>(smem + NW * ST * STAGE);
-  Merge& mg = *reinterpret_cast<Merge*>(smem);                    // aliases the ring
+  // the merge buffers alias the ring; the ring is zeroed again after every merge so that it only
+  // ever holds finite coefficients or zeros
+  static_assert(sizeof(Merge) <= (size_t)NW * ST * STAGE, "merge buffers fit in the ring");
+  Merge& mg = *reinterpret_cast<Merge*>(smem);
   __shared__ long long segW[64];                                  // per-sequence stream length
+  __shared__ uint64_t bar_all[NW * ST];                           // one full-barrier per ring stage
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int g8 = lane >> 2, c = lane & 3;
   const int C = gridDim.x, cta = blockIdx.x;
 
+  // self-contained setup first (it may overlap the tail of the preceding grid)
+  // the ring only ever holds finite coefficients or zeros
+  for (int i = tid; i < NW * ST * STAGE / 16; i += blockDim.x)
+    reinterpret_cast<uint4*>(ring)[i] = make_uint4(0, 0, 0, 0);
+  if (tid < NW * ST) mbar_init(&bar_all[tid], 1);
+  fence_mbar_init();
+  fence_proxy_async_smem();
+  pdl_wait();   // everything below reads data written by earlier grids
   // stream length of every sequence of this layer (same for every head); poisoned tables -> 0
   for (int b = tid; b < s.B; b += blockDim.x) {
     const long long w = bucket_base[((long long)b * s.L + layer) * (kMaxR + 2) + kMaxR + 1];
     segW[b] = (w >= 0 && w <= s.cap) ? w : 0;
   }
-  // the ring only ever holds finite coefficients or zeros
-  for (int i = tid; i < NW * ST * STAGE / 16; i += blockDim.x)
-    reinterpret_cast<uint4*>(ring)[i] = make_uint4(0, 0, 0, 0);
   __syncthreads();
+  uint32_t n_issued = 0;   // chunks this warp has consumed (== index of its next chunk)
+  int n_pending = 0;       // chunks issued but not yet consumed
+  bool timed_out = false;
   long long T = 0;
   for (int b = 0; b < s.B; ++b) T += segW[b] * s.G;
-  if (T == 0) return;
+  if (T == 0) { pdl_trigger(); return; }
   const long long lo_g = (long long)((__int128)T * cta / C);
   const long long hi_g = (long long)((__int128)T * (cta + 1) / C);
 
@@ -228,141 +241,192 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
         if (r <= kMaxR) sm.cnt[r] = bucket_count[bl * (kMaxR + 1) + r];
         sm.base[r] = bucket_base[bl * (kMaxR + 2) + r];
       }
-      rotate_queries(sm, basis_k + ((long long)layer * s.G + g) * kHeadDim * kHeadDim,
-                     qin + ((long long)b * s.H + (long long)g * s.grp) * kHeadDim, s.grp, warp, lane);
       __syncthreads();
-      build_qfrag(sm, tid);
+      for (int r = tid; r <= kMaxR; r += blockDim.x) {
+        long long i0 = 0, i1 = 0;
+        if (r >= s.r_min && r <= s.r_max) bucket_range(sm, r, lo, hi, i0, i1);
+        sm.it_lo[r] = (int)i0;
+        sm.it_pref[r + 1] = (int)(i1 - i0);   // counts first, prefixed below
+      }
       __syncthreads();
-
+      if (tid == 0) {
+        int acc = 0;
+        sm.it_pref[0] = 0;
+        for (int r = 0; r <= kMaxR; ++r) { acc += sm.it_pref[r + 1]; sm.it_pref[r + 1] = acc; }
+      }
+      __syncthreads();
+      // start this warp's loads first: they do not depend on the rotated queries
       const __nv_bfloat16* cK = coef + ((bl * s.G + g) * 2) * s.cap;
       const __nv_bfloat16* cV = cK + s.cap;
       const uint32_t ring_w = smem_addr(ring) + warp * ST * STAGE;
+      uint64_t* bars = &bar_all[warp * ST];
 
       float Mx[2] = {-INFINITY, -INFINITY}, Ls[2] = {0.f, 0.f};
       float oacc[kHeadDim / 16][4];
 #pragma unroll
       for (int t = 0; t < kHeadDim / 16; ++t) oacc[t][0] = oacc[t][1] = oacc[t][2] = oacc[t][3] = 0.f;
 
+      const int total = sm.it_pref[kMaxR + 1];
       Prod pr;
-      pr.items.r = s.r_min - 1; pr.items.it = pr.items.it_end = 0; pr.items.k = 0;
-      pr.live = iter_seek(pr.items, sm, lo, hi, s.r_max, warp);
-      pr.phase = 0; pr.jc = 0;
-      ItemIter cons = pr.items;
-      bool cons_live = pr.live;
-      int stage_p = 0, stage_c = 0;
+      pr.k = warp; pr.phase = 0; pr.jc = 0;
+      if (pr.k < total) pr.item = item_at(sm, pr.k);
+      int cons_k = pr.k;
+      Item cons = pr.item;
 #pragma unroll
-      for (int i = 0; i < ST - 1; ++i) {
-        issue_chunk(pr, sm, cK, cV, ring_w + stage_p * STAGE, lo, hi, s.r_max, warp, lane);
-        stage_p = (stage_p + 1) % ST;
-      }
+      for (int i = 0; i < ST - 1; ++i)
+        if (issue_chunk(pr, sm, cK, cV, ring_w + ((n_issued + i) % ST) * STAGE,
+                        &bars[(n_issued + i) % ST], total, lane)) ++n_pending;
+      rotate_queries(sm, basis_k + ((long long)layer * s.G + g) * kHeadDim * kHeadDim,
+                     qin + ((long long)b * s.H + (long long)g * s.grp) * kHeadDim, s.grp, warp, lane);
+      __syncthreads();
+      build_qfrag(sm, tid);
+      __syncthreads();
 
-      while (cons_live) {
+      // chunk k of this warp (counted over the whole kernel) lives in stage k % ST, phase (k/ST)&1
+
+      auto wait_chunk = [&]() -> bool {
+        const uint32_t k = n_issued;
+        if (!mbar_wait_bounded(&bars[k % ST], (k / ST) & 1u, kWaitTries)) { timed_out = true; return false; }
+        return true;
+      };
+      auto next_chunk = [&]() {
+        // the consumed stage is free again: refill it with the chunk ST-1 ahead
+        ++n_issued;
+        --n_pending;
+        if (issue_chunk(pr, sm, cK, cV, ring_w + ((n_issued + ST - 2) % ST) * STAGE,
+                        &bars[(n_issued + ST - 2) % ST], total, lane)) ++n_pending;
+      };
+
+      while (cons_k < total && !timed_out) {
         const int r = cons.r;
-        const int nj = (r + 15) >> 4;
-        const long long n_real = sm.cnt[r] - cons.it * ISL;   // real slots of this item (may exceed ISL)
+        const int nj = (r + CH - 1) / CH;
+        const long long n_real = sm.cnt[r] - (long long)cons.it * ISL;   // real slots of this item
         float sc[ISL / 16][4];
 #pragma unroll
         for (int t = 0; t < ISL / 16; ++t) sc[t][0] = sc[t][1] = sc[t][2] = sc[t][3] = 0.f;
 
-        // ---- K chunks: scores
+        // ---- K chunks: scores (rows >= r masked in the q~ fragment)
         for (int jc = 0; jc < nj; ++jc) {
-          cp_async_wait<ST - 2>();
-          __syncwarp();
-          const uint32_t st_addr = ring_w + stage_c * STAGE;
-          const uint4 qf = *reinterpret_cast<const uint4*>(&sm.qfrag[jc][lane][0]);
+          if (!wait_chunk()) break;
+          const uint32_t st_addr = ring_w + (n_issued % ST) * STAGE;
           const int m = lane >> 3, r8 = lane & 7;
-          const uint32_t a_base = st_addr + ((m >> 1) * 8 + r8) * ROWB + (m & 1) * 16;
 #pragma unroll
-          for (int mt = 0; mt < ISL / 16; ++mt) {
-            uint32_t a[4];
-            ldsm_x4_trans(a_base + mt * 32, a);
-            mma_bf16_16816(sc[mt], a, qf.x, qf.y);
-            mma_bf16_16816(sc[mt], a, qf.z, qf.w);
+          for (int ks = 0; ks < CH / 16; ++ks) {
+            const int j16 = jc * CH + ks * 16;
+            if (j16 >= r) break;                        // warp-uniform
+            uint4 qf = *reinterpret_cast<const uint4*>(&sm.qfrag[j16 >> 4][lane][0]);
+            const int jb = j16 + 2 * c;
+            qf.x = keep_rows(qf.x, jb, r); qf.z = keep_rows(qf.z, jb, r);
+            qf.y = keep_rows(qf.y, jb + 8, r); qf.w = keep_rows(qf.w, jb + 8, r);
+            const uint32_t a_base = st_addr + (ks * 16 + (m >> 1) * 8 + r8) * ROWB + (m & 1) * 16;
+            uint32_t a[ISL / 16][4];
+#pragma unroll
+            for (int mt = 0; mt < ISL / 16; ++mt) ldsm_x4_trans(a_base + mt * 32, a[mt]);
+#pragma unroll
+            for (int mt = 0; mt < ISL / 16; ++mt) mma_bf16_16816(sc[mt], a[mt], qf.x, qf.y);
+#pragma unroll
+            for (int mt = 0; mt < ISL / 16; ++mt) mma_bf16_16816(sc[mt], a[mt], qf.z, qf.w);
           }
           __syncwarp();
-          issue_chunk(pr, sm, cK, cV, ring_w + stage_p * STAGE, lo, hi, s.r_max, warp, lane);
-          stage_p = (stage_p + 1) % ST;
-          stage_c = (stage_c + 1) % ST;
+          next_chunk();
         }
+        if (timed_out) break;
 
         // ---- online softmax over the item's slots (heads 2c, 2c+1 per lane)
         float mloc[2] = {-INFINITY, -INFINITY};
+        const bool full_item = n_real >= ISL;           // warp-uniform: no slot to mask
 #pragma unroll
         for (int mt = 0; mt < ISL / 16; ++mt) {
-          const int s0 = mt * 16 + g8;
-          if (s0 >= n_real) { sc[mt][0] = sc[mt][1] = -INFINITY; }
-          if (s0 + 8 >= n_real) { sc[mt][2] = sc[mt][3] = -INFINITY; }
+          if (!full_item) {
+            const int s0 = mt * 16 + g8;
+            if (s0 >= n_real) { sc[mt][0] = sc[mt][1] = -INFINITY; }
+            if (s0 + 8 >= n_real) { sc[mt][2] = sc[mt][3] = -INFINITY; }
+          }
           mloc[0] = fmaxf(mloc[0], fmaxf(sc[mt][0], sc[mt][2]));
           mloc[1] = fmaxf(mloc[1], fmaxf(sc[mt][1], sc[mt][3]));
         }
+        // The reference max only moves when some score exceeds it by more than kSlack (log2
+        // units): weights stay <= 2^kSlack, exact after the final normalisation, and the common
+        // case costs one warp vote instead of a shuffle reduction and a rescale.
+        float corr[2] = {1.f, 1.f};
+        if (!__all_sync(0xffffffffu, mloc[0] <= Mx[0] + kSlack && mloc[1] <= Mx[1] + kSlack)) {
 #pragma unroll
-        for (int o = 4; o < 32; o <<= 1) {
-          mloc[0] = fmaxf(mloc[0], __shfl_xor_sync(0xffffffffu, mloc[0], o));
-          mloc[1] = fmaxf(mloc[1], __shfl_xor_sync(0xffffffffu, mloc[1], o));
-        }
-        float corr[2];
+          for (int o = 4; o < 32; o <<= 1) {
+            mloc[0] = fmaxf(mloc[0], __shfl_xor_sync(0xffffffffu, mloc[0], o));
+            mloc[1] = fmaxf(mloc[1], __shfl_xor_sync(0xffffffffu, mloc[1], o));
+          }
 #pragma unroll
-        for (int e = 0; e < 2; ++e) {
-          const float nm = fmaxf(Mx[e], mloc[e]);
-          corr[e] = fast_exp2(Mx[e] - nm);
-          Mx[e] = nm;
+          for (int e = 0; e < 2; ++e) {
+            const float nm = fmaxf(Mx[e], mloc[e]);
+            corr[e] = fast_exp2(Mx[e] - nm);
+            Mx[e] = nm;
+          }
+#pragma unroll
+          for (int t = 0; t < kHeadDim / 16; ++t) {
+            oacc[t][0] *= corr[0]; oacc[t][1] *= corr[1];
+            oacc[t][2] *= corr[0]; oacc[t][3] *= corr[1];
+          }
         }
         float lsum[2] = {0.f, 0.f};
-        uint32_t pb[ISL / 16][4];   // per slot tile: b0 hi, b1 hi, b0 lo, b1 lo
+        uint32_t pb[ISL / 16][2];   // per slot tile: b0, b1 of P^T (bf16)
 #pragma unroll
         for (int mt = 0; mt < ISL / 16; ++mt) {
           const float p0 = fast_exp2(sc[mt][0] - Mx[0]), p1 = fast_exp2(sc[mt][1] - Mx[1]);
           const float p2 = fast_exp2(sc[mt][2] - Mx[0]), p3 = fast_exp2(sc[mt][3] - Mx[1]);
           lsum[0] += p0 + p2;
           lsum[1] += p1 + p3;
-          uint32_t h01, l01, h23, l23;
-          split_bf16(p0, p1, h01, l01);
-          split_bf16(p2, p3, h23, l23);
-          pb[mt][0] = movmatrix_trans(h01);
-          pb[mt][1] = movmatrix_trans(h23);
-          pb[mt][2] = movmatrix_trans(l01);
-          pb[mt][3] = movmatrix_trans(l23);
+          pb[mt][0] = movmatrix_trans(pack_bf16(p0, p1));
+          pb[mt][1] = movmatrix_trans(pack_bf16(p2, p3));
         }
         Ls[0] = Ls[0] * corr[0] + lsum[0];
         Ls[1] = Ls[1] * corr[1] + lsum[1];
-#pragma unroll
-        for (int t = 0; t < kHeadDim / 16; ++t) {
-          oacc[t][0] *= corr[0]; oacc[t][1] *= corr[1];
-          oacc[t][2] *= corr[0]; oacc[t][3] *= corr[1];
-        }
 
-        // ---- V chunks: weighted coefficient rows
+        // ---- V chunks: weighted coefficient rows (rows >= r masked in the A fragment)
 #pragma unroll
-        for (int jc = 0; jc < kHeadDim / 16; ++jc) {
+        for (int jc = 0; jc < kHeadDim / CH; ++jc) {
           if (jc >= nj) break;
-          cp_async_wait<ST - 2>();
-          __syncwarp();
-          const uint32_t st_addr = ring_w + stage_c * STAGE;
+          if (!wait_chunk()) break;
+          const uint32_t st_addr = ring_w + (n_issued % ST) * STAGE;
           const int m = lane >> 3, r8 = lane & 7;
-          const uint32_t a_base = st_addr + ((m & 1) * 8 + r8) * ROWB + (m >> 1) * 16;
 #pragma unroll
-          for (int kt = 0; kt < ISL / 16; ++kt) {
-            uint32_t a[4];
-            ldsm_x4(a_base + kt * 32, a);
-            mma_bf16_16816(oacc[jc], a, pb[kt][0], pb[kt][1]);
-            mma_bf16_16816(oacc[jc], a, pb[kt][2], pb[kt][3]);
+          for (int ks = 0; ks < CH / 16; ++ks) {
+            const int jt = jc * (CH / 16) + ks;         // 16-row tile of o~
+            if (jt * 16 >= r) break;                    // warp-uniform
+            const uint32_t a_base = st_addr + (ks * 16 + (m & 1) * 8 + r8) * ROWB + (m >> 1) * 16;
+            const bool keep0 = jt * 16 + g8 < r, keep1 = jt * 16 + g8 + 8 < r;
+            float t1[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+            for (int kt = 0; kt < ISL / 16; kt += 2) {
+              uint32_t a[4], b[4];
+              ldsm_x4(a_base + kt * 32, a);
+              ldsm_x4(a_base + (kt + 1) * 32, b);
+              if (!keep0) { a[0] = a[2] = 0u; b[0] = b[2] = 0u; }
+              if (!keep1) { a[1] = a[3] = 0u; b[1] = b[3] = 0u; }
+              mma_bf16_16816(oacc[jt], a, pb[kt][0], pb[kt][1]);
+              mma_bf16_16816(t1, b, pb[kt + 1][0], pb[kt + 1][1]);
+            }
+#pragma unroll
+            for (int e = 0; e < 4; ++e) oacc[jt][e] += t1[e];
           }
           __syncwarp();
-          issue_chunk(pr, sm, cK, cV, ring_w + stage_p * STAGE, lo, hi, s.r_max, warp, lane);
-          stage_p = (stage_p + 1) % ST;
-          stage_c = (stage_c + 1) % ST;
+          next_chunk();
         }
-        iter_step(cons);
-        cons_live = iter_seek(cons, sm, lo, hi, s.r_max, warp);
+        cons_k += NW;
+        if (cons_k < total) cons = item_at(sm, cons_k);
       }
-      cp_async_wait<0>();
+      // drain: never leave bulk copies in flight into this ring
+      while (n_pending > 0) {
+        mbar_wait_bounded(&bars[n_issued % ST], (n_issued / ST) & 1u, kWaitTries);
+        ++n_issued;
+        --n_pending;
+      }
 
       // ---- merge the warps of this CTA for this segment
 #pragma unroll
       for (int e = 0; e < 2; ++e)
 #pragma unroll
         for (int o = 4; o < 32; o <<= 1) Ls[e] += __shfl_xor_sync(0xffffffffu, Ls[e], o);
-      __syncthreads();   // every warp is done with its ring
+      __syncthreads();   // every warp has finished this segment
       if (g8 == 0) {
         mg.M[warp][2 * c] = Mx[0]; mg.M[warp][2 * c + 1] = Mx[1];
         mg.L[warp][2 * c] = Ls[0]; mg.L[warp][2 * c + 1] = Ls[1];
@@ -395,10 +459,15 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
         out[h * kPartStride + j] = o;
         if (j == 0) { out[h * kPartStride + kHeadDim] = mx; out[h * kPartStride + kHeadDim + 1] = l; }
       }
-      __syncthreads();   // merge buffers alias the ring of the next segment
-      (void)dev_status;
+      __syncthreads();
+      for (int i = tid; i < NW * ST * STAGE / 16; i += blockDim.x)
+        reinterpret_cast<uint4*>(ring)[i] = make_uint4(0, 0, 0, 0);
+      fence_proxy_async_smem();
+      __syncthreads();
     }
   }
+  if (timed_out && lane == 0) raise_status(dev_status, VARRATE_ERR_TIMEOUT);
+  pdl_trigger();
 }
 
 // grid (G, B), 256 threads: merge the partials of segment (b, g), add the exact tail, rotate back.
@@ -443,13 +512,8 @@ decode_combine_mma_kernel(const float* __restrict__ part, const int64_t* __restr
     while (c1 > c0 && (long long)((__int128)T * c1 / C) > P + W - 1) --c1;
   }
   const float scale = kLog2e * rsqrtf((float)kHeadDim);
-  // per head: global max over partials and tail, then weights
-  if (tid < s.grp) {
-    float mx = -INFINITY;
-    for (int cc = c0; cc <= c1; ++cc) mx = fmaxf(mx, part[((cc + seg) * kHeadsPad + tid) * kPartStride + kHeadDim]);
-    hm[tid] = mx;
-  }
-  // exact tail scores (n_tail <= 64 handled here; larger tails use decode.cu's path)
+  pdl_wait();   // the partials come from the preceding decode grid
+  // exact tail scores (n_tail <= 64 on this path)
   for (int i = warp; i < s.grp * n_tail; i += blockDim.x / 32) {
     const int h = i / n_tail, t = i % n_tail;
     const __nv_bfloat16* tk = tail_k + (((long long)b * s.G + g) * n_tail + t) * kHeadDim;
@@ -461,20 +525,28 @@ decode_combine_mma_kernel(const float* __restrict__ part, const int64_t* __restr
     if (lane == 0) tsc[h][t] = a * scale;
   }
   __syncthreads();
-  if (tid < s.grp) {
-    float mx = hm[tid];
-    for (int t = 0; t < n_tail; ++t) mx = fmaxf(mx, tsc[tid][t]);
+  // per head (one warp each): max over partials and tail, then the softmax denominator
+  for (int h = warp; h < s.grp; h += blockDim.x / 32) {
+    float mx = -INFINITY;
+    for (int cc = c0 + lane; cc <= c1; cc += 32)
+      mx = fmaxf(mx, part[((cc + seg) * kHeadsPad + h) * kPartStride + kHeadDim]);
+    for (int t = lane; t < n_tail; t += 32) mx = fmaxf(mx, tsc[h][t]);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
     float l = 0.f;
-    for (int cc = c0; cc <= c1; ++cc) {
-      const float* pp = part + ((cc + seg) * kHeadsPad + tid) * kPartStride;
+    for (int cc = c0 + lane; cc <= c1; cc += 32) {
+      const float* pp = part + ((cc + seg) * kHeadsPad + h) * kPartStride;
       if (pp[kHeadDim] != -INFINITY) l = fmaf(pp[kHeadDim + 1], exp2f(pp[kHeadDim] - mx), l);
     }
-    for (int t = 0; t < n_tail; ++t) {
-      tsc[tid][t] = exp2f(tsc[tid][t] - mx);
-      l += tsc[tid][t];
+    __syncwarp();
+    for (int t = lane; t < n_tail; t += 32) {
+      const float w = exp2f(tsc[h][t] - mx);
+      tsc[h][t] = w;
+      l += w;
     }
-    hm[tid] = mx;
-    hl[tid] = l;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
+    if (lane == 0) { hm[h] = mx; hl[h] = l; }
   }
   __syncthreads();
   for (int i = tid; i < s.grp * kHeadDim; i += blockDim.x) {
@@ -496,6 +568,7 @@ decode_combine_mma_kernel(const float* __restrict__ part, const int64_t* __restr
       y = fmaf(tsc[h][t], __bfloat162float(tail_v[(((long long)b * s.G + g) * n_tail + t) * kHeadDim + col]), y);
     out[((long long)b * s.H + (long long)g * s.grp + h) * kHeadDim + col] = __float2bfloat16_rn(y / hl[h]);
   }
+  pdl_trigger();
 }
 
 }  // namespace
@@ -507,7 +580,7 @@ size_t decode_mma_part_bytes(const Shape& s, int num_sms) {
 }
 
 bool decode_mma_supported(const Shape& s, int n_tail) {
-  return s.dtype == VARRATE_BF16 && s.B <= 64 && n_tail <= 64 && sizeof(Merge) <= (size_t)NW * ST * STAGE;
+  return s.dtype == VARRATE_BF16 && s.B <= 64 && n_tail <= 64;
 }
 
 int launch_decode_mma(const Shape& s, const varrate_packed& c, const void* basis_k,
@@ -516,13 +589,28 @@ int launch_decode_mma(const Shape& s, const varrate_packed& c, const void* basis
                       int num_sms, cudaStream_t st) {
   const size_t smem = decode_mma_smem_bytes();
   cudaFuncSetAttribute(decode_mma_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  decode_mma_kernel<<<num_sms, NW * 32, smem, st>>>(
-      (const __nv_bfloat16*)c.coef, c.bucket_count, c.bucket_base, (const __nv_bfloat16*)basis_k,
-      (const __nv_bfloat16*)q, part, dev_status, s, layer);
-  decode_combine_mma_kernel<<<dim3(s.G, s.B), 256, 0, st>>>(
-      part, c.bucket_base, (const __nv_bfloat16*)q, (const __nv_bfloat16*)basis_v,
-      (const __nv_bfloat16*)tail_k, (const __nv_bfloat16*)tail_v, n_tail, (__nv_bfloat16*)out, s,
-      layer, num_sms);
+  // both grids may be scheduled while their predecessor drains (programmatic dependent launch);
+  // each waits on griddepcontrol.wait before touching what its predecessor wrote
+  cudaLaunchAttribute pdl[1];
+  pdl[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  pdl[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t lc = {};
+  lc.gridDim = dim3(num_sms);
+  lc.blockDim = dim3(NW * 32);
+  lc.dynamicSmemBytes = smem;
+  lc.stream = st;
+  lc.attrs = pdl;
+  lc.numAttrs = 1;
+  cudaLaunchKernelEx(&lc, decode_mma_kernel, (const __nv_bfloat16*)c.coef, (const int32_t*)c.bucket_count,
+                     (const int64_t*)c.bucket_base, (const __nv_bfloat16*)basis_k,
+                     (const __nv_bfloat16*)q, part, dev_status, s, layer);
+  lc.gridDim = dim3(s.G, s.B);
+  lc.blockDim = dim3(256);
+  lc.dynamicSmemBytes = 0;
+  cudaLaunchKernelEx(&lc, decode_combine_mma_kernel, (const float*)part, (const int64_t*)c.bucket_base,
+                     (const __nv_bfloat16*)q, (const __nv_bfloat16*)basis_v,
+                     (const __nv_bfloat16*)tail_k, (const __nv_bfloat16*)tail_v, n_tail,
+                     (__nv_bfloat16*)out, s, layer, num_sms);
   return 2;
 }
 

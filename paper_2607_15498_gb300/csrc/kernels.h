@@ -21,7 +21,13 @@ SalPlan salience_plan(const Shape& s, int num_sms);
 size_t salience_ws_bytes(const Shape& s, int num_sms);
 // Returns the number of kernels launched.
 int launch_salience(const Shape& s, const void* q_win, const void* k, float* sal_out, void* ws,
-                    int num_sms, cudaStream_t st);
+                    int32_t* dev_status, int num_sms, cudaStream_t st);
+// bf16 tensor-core salience (salience_tc.cu); returns -1 if a TMA descriptor cannot be built
+bool salience_tc_supported(const Shape& s);
+SalPlan salience_tc_plan(const Shape& s, int num_sms);
+size_t salience_tc_ws_bytes(const Shape& s, int num_sms);
+int launch_salience_tc(const Shape& s, const void* q_win, const void* k, float* sal_out, void* ws,
+                       int32_t* dev_status, int num_sms, cudaStream_t st);
 
 // ---- step 2: allocation
 int launch_allocate(const Shape& s, const float* sal, uint8_t* ranks, int64_t* realized,

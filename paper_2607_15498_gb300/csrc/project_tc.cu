@@ -3,9 +3,11 @@
 // the rank-bucketed layout.
 //
 // One CTA (4 warps) owns a range of bucketed slots of one (sequence, layer, head, K-or-V) stream.
-//   gather   thread i copies token perm[slot0 + i] (256 B) into row i of a 128 x 128 bf16 tile
-//            with 16-byte cp.async, already in the K-major 128-byte-swizzled layout the tensor
-//            core reads; 4 stages, 3 tiles in flight.
+//   gather   token perm[slot0 + i] (256 B) goes to row i of a 128 x 128 bf16 tile with 16-byte
+//            cp.async (16 lanes per row, so one warp instruction moves two whole rows), already in
+//            the K-major 128-byte-swizzled layout the tensor core reads; 5 stages, 4 tiles in flight. Tokens sit in slot order inside a bucket, so
+//            the slot alone gives the rank (prefix search over bucket counts) and the position
+//            (slot - bucket start); only perm is read, one tile ahead of its gather.
 //   mma      one thread issues 8 x tcgen05.mma (M = 128 slots, N = 128 coefficients, K = 16) with
 //            U (128 x 128, resident in shared memory) as B; fp32 accumulator in TMEM, two
 //            128-column buffers so tile i's MMA overlaps tile i-1's epilogue; completion through
@@ -22,7 +24,7 @@ namespace {
 
 constexpr int kMaxR = kHeadDim;
 constexpr int TM = 128;                    // slots per tile
-constexpr int NST = 4;                     // gather stages
+constexpr int NST = 5;                     // gather stages
 constexpr int TILE_BYTES = TM * kHeadDim * 2;
 constexpr uint32_t kWaitTries = 1u << 22;  // bounded mbarrier polls
 
@@ -34,15 +36,15 @@ struct ProjSmem {
   int rk[NST][TM];
   int ps[NST][TM];
   int n8[kMaxR + 1];
+  int slot_start[kMaxR + 2];   // first bucketed slot of rank r (exclusive prefix of the counts)
   long long base[kMaxR + 2];
 };
 
 __global__ void __launch_bounds__(128, 1)
 project_tc_kernel(const __nv_bfloat16* __restrict__ k, const __nv_bfloat16* __restrict__ v,
                   const __nv_bfloat16* __restrict__ basis_k, const __nv_bfloat16* __restrict__ basis_v,
-                  const uint8_t* __restrict__ ranks, const int32_t* __restrict__ bucket_count,
-                  const int64_t* __restrict__ bucket_base, const int32_t* __restrict__ perm,
-                  const int32_t* __restrict__ pos, __nv_bfloat16* __restrict__ coef,
+                  const int32_t* __restrict__ bucket_count, const int64_t* __restrict__ bucket_base,
+                  const int32_t* __restrict__ perm, __nv_bfloat16* __restrict__ coef,
                   int32_t* __restrict__ dev_status, Shape s, int64_t chunk) {
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   // 1024-byte alignment for the swizzled operand tiles
@@ -60,7 +62,15 @@ project_tc_kernel(const __nv_bfloat16* __restrict__ k, const __nv_bfloat16* __re
     if (r <= kMaxR) sm.n8[r] = (int)pad8(bucket_count[bl * (kMaxR + 1) + r]);
     sm.base[r] = bucket_base[bl * (kMaxR + 2) + r];
   }
-  if (tid == 0) sm.err = 0;
+  if (tid == 0) {
+    sm.err = 0;
+    int acc = 0;
+    for (int r = 0; r <= kMaxR; ++r) {
+      sm.slot_start[r] = acc;
+      acc += bucket_count[bl * (kMaxR + 1) + r];
+    }
+    sm.slot_start[kMaxR + 1] = acc;
+  }
   __syncthreads();
   if (sm.base[kMaxR + 1] > s.cap || sm.base[kMaxR + 1] < 0) return;   // reported by pack_tables
 
@@ -92,23 +102,44 @@ project_tc_kernel(const __nv_bfloat16* __restrict__ k, const __nv_bfloat16* __re
   const uint32_t stage0 = smem_addr(stages), u_addr = smem_addr(u_tile);
   constexpr uint32_t idesc = idesc_bf16_f32(TM, kHeadDim);
 
+  // perm of the next tile to gather, loaded one iteration ahead (-1 past the range)
+  auto perm_of = [&](int i) -> int {
+    const int64_t slot = s_begin + (int64_t)i * TM + tid;
+    return (i < n_tiles && slot < s_end) ? perm[bl * s.N + slot] : -1;
+  };
+  // slot metadata of row `tid` of tile i (token, rank, position in bucket) into its stage
+  auto stage_meta = [&](int i, int t) {
+    if (i >= n_tiles) return;
+    const int st = i % NST;
+    const int slot = (int)(s_begin + (int64_t)i * TM + tid);
+    int r = 0, p = 0;
+    if (t >= 0) {
+      int lo = 0, hi = kMaxR + 1;   // slot_start[lo] <= slot < slot_start[hi]
+      while (hi - lo > 1) {
+        const int mid = (lo + hi) >> 1;
+        if (sm.slot_start[mid] <= slot) lo = mid; else hi = mid;
+      }
+      r = lo;
+      p = slot - sm.slot_start[lo];
+    }
+    sm.tok[st][tid] = t;
+    sm.rk[st][tid] = r;
+    sm.ps[st][tid] = p;
+  };
+  // copies of tile i (after its metadata is visible): 16 lanes per 256-byte row, so one warp
+  // instruction moves two whole rows
   auto gather = [&](int i) {
     if (i < n_tiles) {
       const int st = i % NST;
-      const int64_t slot = s_begin + (int64_t)i * TM + tid;
-      int t = -1, r = 0, p = 0;
-      if (slot < s_end) {
-        t = perm[bl * s.N + slot];
-        r = ranks[bl * s.N + t];
-        p = pos[bl * s.N + t];
-      }
-      sm.tok[st][tid] = t;
-      sm.rk[st][tid] = r;
-      sm.ps[st][tid] = p;
-      const __nv_bfloat16* src = x + (int64_t)(t < 0 ? 0 : t) * kHeadDim;
       const uint32_t dst = stage0 + st * TILE_BYTES;
+      const int c = tid & 15;
 #pragma unroll
-      for (int c = 0; c < 16; ++c) cp_async16(dst + sw128_offset(tid, c, TM), src + c * 8, t >= 0 ? 16u : 0u);
+      for (int q = 0; q < TM / 8; ++q) {
+        const int row = (tid >> 4) + 8 * q;
+        const int t = sm.tok[st][row];
+        const __nv_bfloat16* src = x + (int64_t)(t < 0 ? 0 : t) * kHeadDim + c * 8;
+        cp_async16(dst + sw128_offset(row, c, TM), src, t >= 0 ? 16u : 0u);
+      }
     }
     cp_async_commit();
   };
@@ -139,6 +170,10 @@ project_tc_kernel(const __nv_bfloat16* __restrict__ k, const __nv_bfloat16* __re
   };
 
 #pragma unroll
+  for (int i = 0; i < NST - 1; ++i) stage_meta(i, perm_of(i));
+  int t_next = perm_of(NST - 1);
+  __syncthreads();
+#pragma unroll
   for (int i = 0; i < NST - 1; ++i) gather(i);
   for (int i = 0; i < n_tiles; ++i) {
     cp_async_wait<NST - 2>();
@@ -156,6 +191,9 @@ project_tc_kernel(const __nv_bfloat16* __restrict__ k, const __nv_bfloat16* __re
       tc_commit(&sm.mma_bar[i & 1]);
     }
     if (i >= 1) epilogue(i - 1);
+    // tile i + NST - 1 reuses the stage of tile i - 1, whose MMA and epilogue are complete
+    stage_meta(i + NST - 1, t_next);
+    t_next = perm_of(i + NST);
     tc_fence_before();
     __syncthreads();
     gather(i + NST - 1);
@@ -184,8 +222,8 @@ int launch_project_tc(const Shape& s, const void* k, const void* v, const void* 
   cudaFuncSetAttribute(project_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   project_tc_kernel<<<dim3(n_chunks, s.G * 2, s.B * s.L), 128, smem, st>>>(
       (const __nv_bfloat16*)k, (const __nv_bfloat16*)v, (const __nv_bfloat16*)basis_k,
-      (const __nv_bfloat16*)basis_v, out.ranks, out.bucket_count, out.bucket_base, out.perm,
-      out.pos, (__nv_bfloat16*)out.coef, dev_status, s, chunk);
+      (const __nv_bfloat16*)basis_v, out.bucket_count, out.bucket_base, out.perm,
+      (__nv_bfloat16*)out.coef, dev_status, s, chunk);
   return 1;
 }
 

@@ -232,6 +232,7 @@ __global__ void salience_pool_kernel(const float* __restrict__ raw, float* __res
 }  // namespace
 
 size_t salience_ws_bytes(const Shape& s, int num_sms) {
+  if (salience_tc_supported(s)) return salience_tc_ws_bytes(s, num_sms);
   const SalPlan p = salience_plan(s, num_sms);
   const int M = s.grp * s.w;
   size_t b = (size_t)s.B * s.L * s.G * M * p.n_chunks * sizeof(float2);
@@ -260,7 +261,8 @@ SalPlan salience_plan(const Shape& s, int num_sms) {
 }
 
 int launch_salience(const Shape& s, const void* q_win, const void* k, float* sal_out, void* ws,
-                    int num_sms, cudaStream_t st) {
+                    int32_t* dev_status, int num_sms, cudaStream_t st) {
+  if (salience_tc_supported(s)) return launch_salience_tc(s, q_win, k, sal_out, ws, dev_status, num_sms, st);
   const SalPlan p = salience_plan(s, num_sms);
   if (s.n_coded == 0) return 0;
   const int M = s.grp * s.w;
