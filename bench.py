@@ -52,6 +52,25 @@ def measured_peaks():
     return FALLBACK_HBM_GBS, "fallback"
 
 
+def measured_traffic():
+    """DRAM bytes (read + write) per launch of the decode kernel from the committed ncu summary, or
+    None when that summary was taken on a different version of the kernel source."""
+    import hashlib
+    import re
+    prof = os.path.join(ROOT, "profiles", "decode_mma_llama32.md")
+    src = os.path.join(ROOT, "paper_2607_15498_gb300", "csrc", "decode_mma.cu")
+    if not (os.path.exists(prof) and os.path.exists(src)):
+        return None
+    text = open(prof).read()
+    m_bytes = re.search(r"traffic_bytes_per_launch:\s*([0-9]+)", text)
+    m_sha = re.search(r"kernel_source_sha256:\s*([0-9a-f]{64})", text)
+    if not (m_bytes and m_sha):
+        return None
+    if hashlib.sha256(open(src, "rb").read()).hexdigest() != m_sha.group(1):
+        return None
+    return int(m_bytes.group(1))
+
+
 def dist_env():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -405,7 +424,7 @@ def main():
                 decode_frac_of_nominal_8tbs=round(dec_gbs / world / 8000.0, 4),
                 roofline={"bound": "hbm", "kernel": "varrate_decode_attn (rotate + split + combine)",
                           "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
-                          "frac": round(achieved / peak, 4), "traffic": None,
+                          "frac": round(achieved / peak, 4), "traffic": measured_traffic(),
                           "peak_source": f"{peak_kind} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)"
                           if peak_kind == "measured" else "fallback 6.8 TB/s",
                           "bytes_per_launch": int(bytes_per_call),

@@ -78,11 +78,17 @@ typedef struct {
  *
  * For each (sequence b, layer l) one bucket table, shared by every KV head and by K and V, groups
  * the tokens by rank. With n_r tokens of rank r and n8_r = n_r rounded up to a multiple of 8:
- *   bucket_base[r_min] = 0, bucket_base[r + 1] = bucket_base[r] + r * n8_r,
- * and coefficient j (< r_t) of token t of stream (b, l, g, kv) sits at element
- *   coef[(((b * L + l) * G + g) * 2 + kv) * cap_elems + bucket_base[r_t] + j * n8_{r_t} + pos[t]]
- * (coefficient-major inside a bucket: one coefficient of consecutive tokens is contiguous).
- * Padding slots pos in [n_r, n8_r) hold zeros. kv = 0 is K, 1 is V. */
+ *   bucket_base[r_min] = 0, bucket_base[r + 1] = bucket_base[r] + r * n8_r.
+ * Bucket r's slots p in [0, n8_r) (token perm-order; p = pos[t]) are cut into tiles of 128 slots,
+ * the last one holding tl = n8_r - 128 i slots. Tile i stores r rows of tl elements back to back,
+ * one row per coefficient, from element bucket_base[r] + 128 i r; in row j the group of 8 slots
+ * g = (p mod 128) / 8 sits at position (g + j) mod (tl / 8). So coefficient j (< r_t) of token t of
+ * stream (b, l, g, kv) is at element
+ *   coef[(((b * L + l) * G + g) * 2 + kv) * cap_elems + bucket_base[r] + 128 i r + j * tl
+ *        + 8 * ((g + j) mod (tl / 8)) + p mod 8],   i = p / 128, r = r_t, p = pos[t].
+ * Every tile, and every run of its rows, is one contiguous block (one bulk copy); the rotation keeps
+ * a block copied verbatim to shared memory free of bank conflicts. Padding slots p in [n_r, n8_r)
+ * hold zeros. kv = 0 is K, 1 is V. */
 typedef struct {
   void* coef;             /* [B][L][G][2][cap_elems] dtype */
   int32_t* bucket_count;  /* [B][L][d + 1]  n_r (0 for r < r_min) */

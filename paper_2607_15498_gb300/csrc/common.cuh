@@ -253,3 +253,22 @@ namespace vr {
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;\n" ::: "memory"); }
 __device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory"); }
 }  // namespace vr
+
+namespace vr {
+// Packed layout inside one rank bucket (n8 slots, rank r, bucket start base_r): slots are cut into
+// tiles of 128 (the last one shorter, tl = min(128, n8 - 128 i)). Tile i holds r rows of tl
+// elements, one row per coefficient, rows back to back, starting at base_r + 128 i r; inside row j
+// the 8-slot groups are rotated by j (group g is stored at position (g + j) mod (tl / 8)), so that a
+// tile (or any run of its rows) is one contiguous block and 8 consecutive rows of one slot group sit
+// in 8 different shared-memory bank groups once the block is copied verbatim.
+__host__ __device__ __forceinline__ long long coef_offset(int r, long long n8, long long p, int j) {
+  const long long t0 = (p >> 7) << 7;
+  const long long rem = n8 - t0;
+  const int tl = (int)(rem < 128 ? rem : 128);
+  const int ng = tl >> 3;
+  const int pl = (int)(p - t0);
+  int grp = (pl >> 3) + j;
+  grp = (ng == 16) ? (grp & 15) : (grp % ng);
+  return t0 * r + (long long)j * tl + grp * 8 + (pl & 7);
+}
+}  // namespace vr

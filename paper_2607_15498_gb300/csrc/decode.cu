@@ -6,10 +6,9 @@
 //
 // decode_rotate  q~ for every head (fp32 workspace).
 // decode_split   grid (S, G, B), 8 warps. The coded elements of the (b, l, g) stream are split
-//                into S contiguous cost ranges; a warp item is 256 consecutive slots of one rank
-//                bucket (8 slots per lane, one 16-byte load per coefficient row). Both K and V are
-//                coefficient-major inside a bucket, so every load is a coalesced 512-byte warp
-//                row. Scores: 8 slots x GP heads per lane, no cross-lane work. Value rows: every
+//                into S contiguous cost ranges; a warp item is one 128-slot tile of a rank bucket
+//                (8 slots per lane on 16 lanes, one 16-byte load per coefficient row, addressed
+//                through the packed layout's coef_offset). Scores: 8 slots x GP heads per lane, no cross-lane work. Value rows: every
 //                lane forms GP x RG partial sums (GP heads x RG rows, GP * RG = 32) and one
 //                31-shuffle transpose-reduction leaves lane i with the full sum of pair i, so each
 //                lane owns 128 / RG output coordinates. Online softmax per warp; warps then merge
@@ -24,7 +23,7 @@ namespace {
 
 constexpr int kMaxR = kHeadDim;
 constexpr int kWarps = 8;
-constexpr int kItem = 256;        // slots per warp item
+constexpr int kItem = 128;        // slots per warp item: one tile of the packed layout
 constexpr int kMaxTail = 4096;
 
 // Raw 8-element row fragment: bf16 -> one uint4, fp32 -> two float4.
@@ -145,9 +144,9 @@ decode_split_kernel(const T* __restrict__ coef, const int32_t* __restrict__ buck
     for (long long it = i_lo; it < i_hi; ++it, ++counter) {
       if ((counter % kWarps) != warp) continue;
       const long long s0 = it * kItem + lane * 8;
-      const bool lane_ok = s0 < n8;
-      const T* kp = cK + b0 + s0;
-      const T* vp = cV + b0 + s0;
+      const bool lane_ok = lane < kItem / 8 && s0 < n8;   // lanes 16..31 idle: 8 slots per lane
+      const T* kp = cK + b0;
+      const T* vp = cV + b0;
 
       // scores for 8 slots x GP heads
       float sc[GP][8];
@@ -159,7 +158,7 @@ decode_split_kernel(const T* __restrict__ coef, const int32_t* __restrict__ buck
         Frag<T> f[8];
 #pragma unroll
         for (int jj = 0; jj < 8; ++jj) {
-          if (lane_ok && j0 + jj < r) f[jj].load(kp + (long long)(j0 + jj) * n8);
+          if (lane_ok && j0 + jj < r) f[jj].load(kp + coef_offset(r, n8, s0, j0 + jj));
           else f[jj].zero();
         }
 #pragma unroll
@@ -210,7 +209,7 @@ decode_split_kernel(const T* __restrict__ coef, const int32_t* __restrict__ buck
         Frag<T> f[RG];
 #pragma unroll
         for (int jj = 0; jj < RG; ++jj) {
-          if (lane_ok && gi * RG + jj < r) f[jj].load(vp + (long long)(gi * RG + jj) * n8);
+          if (lane_ok && gi * RG + jj < r) f[jj].load(vp + coef_offset(r, n8, s0, gi * RG + jj));
           else f[jj].zero();
         }
         float pv[32];

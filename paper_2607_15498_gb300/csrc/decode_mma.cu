@@ -8,12 +8,14 @@
 // line (element offsets, K stream); the persistent grid (one CTA per SM) cuts it into equal
 // ranges, so every SM moves the same number of bytes. A CTA walks the (sequence, head) segments its
 // range touches; per segment it rotates the query with mma.sync (U_K tile x q), then its warps take
-// 128-slot items of one rank bucket round-robin. An item of rank r is 2 * ceil(r/32) chunks of 32
-// coefficient rows x 128 slots (8 KB): all K chunks, then all V chunks.
+// 128-slot items (one tile of the packed layout) of one rank bucket round-robin. An item of rank r
+// is 2 * ceil(r/32) chunks of up to 32 coefficient rows x 128 slots (8 KB), each one contiguous
+// block: all K chunks, then all V chunks.
 //
-// Memory path. Each warp owns a 3-stage shared-memory ring filled by 1-D TMA bulk copies (one per
-// coefficient row, one lane per row) that complete on a per-stage mbarrier; the warp stays 2 chunks
-// ahead of the chunk it computes on, across item boundaries, so loads never wait on arithmetic. Rows >= r of a chunk are never loaded; they are masked out of the tensor-core
+// Memory path. Each warp owns a 3-stage shared-memory ring filled by one 1-D TMA bulk copy per
+// chunk that completes on a per-stage mbarrier; the warp stays 2 chunks ahead of the chunk it
+// computes on, across item boundaries, so loads never wait on arithmetic. The per-row rotation of
+// the 8-slot groups keeps the unpadded staged rows free of shared-memory bank conflicts. Rows >= r of a chunk are never loaded; they are masked out of the tensor-core
 // fragments instead, and the ring only ever holds finite coefficients.
 //
 // Arithmetic (per warp, fp32 accumulate, all operands exact or split hi+lo in bf16):
@@ -38,8 +40,7 @@ constexpr int NW = 8;                 // warps per CTA
 constexpr int ST = 3;                 // ring stages per warp
 constexpr int ISL = 128;              // slots per item
 constexpr int CH = 32;                // coefficient rows per chunk
-constexpr int ROWB = ISL * 2 + 16;    // bytes per staged row (+16 B: conflict-free ldmatrix)
-constexpr int STAGE = CH * ROWB;      // one chunk: 32 rows
+constexpr int STAGE = CH * ISL * 2;   // one chunk: up to 32 rows of a 128-slot tile
 constexpr int kPartStride = kHeadDim + 2;
 constexpr int kHeadsPad = 8;
 constexpr uint32_t kWaitTries = 1u << 22;   // bounded mbarrier polls (well over a second)
@@ -100,7 +101,8 @@ struct Prod {
   int jc;      // 16-row chunk index
 };
 
-// Issue the next chunk of this warp's stream into `stage` (one lane per row).
+// Issue the next chunk of this warp's stream into `stage`: rows j0..j0+31 of one 128-slot tile are
+// contiguous in the packed layout, so one bulk copy moves the whole chunk.
 // Returns false (and issues nothing) when the stream is exhausted.
 __device__ __forceinline__ bool issue_chunk(Prod& p, const SegSmem& sm, const __nv_bfloat16* cK,
                                             const __nv_bfloat16* cV, uint32_t stage_addr,
@@ -108,16 +110,16 @@ __device__ __forceinline__ bool issue_chunk(Prod& p, const SegSmem& sm, const __
   if (p.k >= total) return false;
   const int r = p.item.r;
   const long long n8 = pad8(sm.cnt[r]);
-  const long long s_begin = (long long)p.item.it * ISL;
-  const uint32_t row_bytes = (uint32_t)min((long long)ISL, n8 - s_begin) * 2u;   // multiple of 16
+  const long long t0 = (long long)p.item.it * ISL;            // first slot of the tile
+  const long long tl = min((long long)ISL, n8 - t0);            // slots in the tile (multiple of 8)
   const int j0 = p.jc * CH;
   const int rows = min(CH, r - j0);
-  if (lane == 0) mbar_arrive_expect_tx(bar, row_bytes * (uint32_t)rows);
-  __syncwarp();
-  fence_proxy_async_smem();   // earlier ldmatrix reads of this stage precede the async writes
-  if (lane < rows) {
-    const __nv_bfloat16* src = (p.phase ? cV : cK) + sm.base[r] + (long long)(j0 + lane) * n8 + s_begin;
-    bulk_g2s(stage_addr + lane * ROWB, src, row_bytes, bar);
+  // callers have __syncwarp()ed: every lane's ldmatrix reads of this stage are done
+  if (lane == 0) {
+    const uint32_t bytes = (uint32_t)(rows * tl * 2);           // rows j0.. of the tile: contiguous
+    mbar_arrive_expect_tx(bar, bytes);
+    fence_proxy_async_smem();  // the generic reads above precede the async write
+    bulk_g2s(stage_addr, (p.phase ? cV : cK) + sm.base[r] + t0 * r + (long long)j0 * tl, bytes, bar);
   }
   const int nj = (r + CH - 1) / CH;
   if (++p.jc == nj) {
@@ -129,6 +131,14 @@ __device__ __forceinline__ bool issue_chunk(Prod& p, const SegSmem& sm, const __
     }
   }
   return true;
+}
+
+// (x + 2) mod n for 0 <= x < n, n >= 1
+__device__ __forceinline__ int wrap2(int x, int n) {
+  x += 2;
+  x -= (x >= n) ? n : 0;
+  x -= (x >= n) ? n : 0;
+  return x;
 }
 
 // Keep the bf16 halves of `w` whose row index (lo half: j, hi half: j + 1) is below r.
@@ -301,6 +311,11 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
         const int r = cons.r;
         const int nj = (r + CH - 1) / CH;
         const long long n_real = sm.cnt[r] - (long long)cons.it * ISL;   // real slots of this item
+        // tile geometry (packed layout, coef_offset): rows of tl slots, 8-slot group g of row j
+        // stored at position (g + j) mod (tl / 8)
+        const int tl = (int)min((long long)ISL, pad8(sm.cnt[r]) - (long long)cons.it * ISL);
+        const int ng = tl >> 3;
+        const uint32_t row_bytes = (uint32_t)tl * 2u;
         float sc[ISL / 16][4];
 #pragma unroll
         for (int t = 0; t < ISL / 16; ++t) sc[t][0] = sc[t][1] = sc[t][2] = sc[t][3] = 0.f;
@@ -318,10 +333,17 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
             const int jb = j16 + 2 * c;
             qf.x = keep_rows(qf.x, jb, r); qf.z = keep_rows(qf.z, jb, r);
             qf.y = keep_rows(qf.y, jb + 8, r); qf.w = keep_rows(qf.w, jb + 8, r);
-            const uint32_t a_base = st_addr + (ks * 16 + (m >> 1) * 8 + r8) * ROWB + (m & 1) * 16;
+            // this lane's row of the 8x8 matrices: coefficient j, staged at row (j - chunk start)
+            const int jrow = ks * 16 + (m >> 1) * 8 + r8;
+            const int j = jc * CH + jrow;
+            const uint32_t row_addr = st_addr + jrow * row_bytes;
             uint32_t a[ISL / 16][4];
+            int pg = ((m & 1) + j) % ng;                // stored position of slot group 2 mt + (m & 1)
 #pragma unroll
-            for (int mt = 0; mt < ISL / 16; ++mt) ldsm_x4_trans(a_base + mt * 32, a[mt]);
+            for (int mt = 0; mt < ISL / 16; ++mt) {
+              ldsm_x4_trans(row_addr + 16 * pg, a[mt]);
+              pg = wrap2(pg, ng);
+            }
 #pragma unroll
             for (int mt = 0; mt < ISL / 16; ++mt) mma_bf16_16816(sc[mt], a[mt], qf.x, qf.y);
 #pragma unroll
@@ -392,14 +414,19 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
           for (int ks = 0; ks < CH / 16; ++ks) {
             const int jt = jc * (CH / 16) + ks;         // 16-row tile of o~
             if (jt * 16 >= r) break;                    // warp-uniform
-            const uint32_t a_base = st_addr + (ks * 16 + (m & 1) * 8 + r8) * ROWB + (m >> 1) * 16;
+            const int jrow = ks * 16 + (m & 1) * 8 + r8;
+            const int j = jc * CH + jrow;
+            const uint32_t row_addr = st_addr + jrow * row_bytes;
             const bool keep0 = jt * 16 + g8 < r, keep1 = jt * 16 + g8 + 8 < r;
             float t1[4] = {0.f, 0.f, 0.f, 0.f};
+            int pg = ((m >> 1) + j) % ng;               // stored position of slot group 2 kt + (m >> 1)
 #pragma unroll
             for (int kt = 0; kt < ISL / 16; kt += 2) {
               uint32_t a[4], b[4];
-              ldsm_x4(a_base + kt * 32, a);
-              ldsm_x4(a_base + (kt + 1) * 32, b);
+              ldsm_x4(row_addr + 16 * pg, a);
+              pg = wrap2(pg, ng);
+              ldsm_x4(row_addr + 16 * pg, b);
+              pg = wrap2(pg, ng);
               if (!keep0) { a[0] = a[2] = 0u; b[0] = b[2] = 0u; }
               if (!keep1) { a[1] = a[3] = 0u; b[1] = b[3] = 0u; }
               mma_bf16_16816(oacc[jt], a, pb[kt][0], pb[kt][1]);

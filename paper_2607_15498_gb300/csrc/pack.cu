@@ -9,7 +9,8 @@
 //   perm[slot]         token of each slot, buckets in increasing rank;
 //   pad slots          [count[r], pad8(count[r])) of every bucket of every stream set to 0.
 // project (grid over slot chunks x (head, K/V) x (sequence, layer)): tokens are visited in
-// bucketed slot order, so one coefficient of consecutive slots lands on consecutive addresses.
+// bucketed slot order, so one coefficient of consecutive slots lands in consecutive addresses of
+// its 8-slot group (layout: coef_offset in common.cuh).
 #include "common.cuh"
 #include "kernels.h"
 
@@ -110,7 +111,7 @@ pack_tables_kernel(const uint8_t* __restrict__ ranks, int32_t* __restrict__ buck
     for (int64_t i = tid; i < n_streams * per_stream; i += blockDim.x) {
       const int64_t st = i / per_stream, rem = i % per_stream;
       const int64_t j = rem / npad, p = n + rem % npad;
-      coef[(bl * n_streams + st) * s.cap + base[r] + j * n8 + p] = from_f<T>(0.f);
+      coef[(bl * n_streams + st) * s.cap + base[r] + coef_offset(r, n8, p, (int)j)] = from_f<T>(0.f);
     }
   }
 }
@@ -203,7 +204,7 @@ project_kernel(const T* __restrict__ k, const T* __restrict__ v, const T* __rest
       const int slot = i % kTile, j = i / kTile;
       const int r = srk[slot];
       if (stok[slot] >= 0 && j < r)
-        out[bases[r] + (int64_t)j * n8s[r] + spos[slot]] = from_f<T>(xs[slot * kLd + j]);
+        out[bases[r] + coef_offset(r, n8s[r], spos[slot], j)] = from_f<T>(xs[slot * kLd + j]);
     }
   }
 }

@@ -2,19 +2,22 @@
 // (Algorithm 1's projection c_t = U x_t, Eq. 5 with the anchor mean at 0), written straight into
 // the rank-bucketed layout.
 //
-// One CTA (4 warps) owns a range of bucketed slots of one (sequence, layer, head, K-or-V) stream.
-//   gather   token perm[slot0 + i] (256 B) goes to row i of a 128 x 128 bf16 tile with 16-byte
-//            cp.async (16 lanes per row, so one warp instruction moves two whole rows), already in
-//            the K-major 128-byte-swizzled layout the tensor core reads; 5 stages, 4 tiles in flight. Tokens sit in slot order inside a bucket, so
-//            the slot alone gives the rank (prefix search over bucket counts) and the position
-//            (slot - bucket start); only perm is read, one tile ahead of its gather.
-//   mma      one thread issues 8 x tcgen05.mma (M = 128 slots, N = 128 coefficients, K = 16) with
-//            U (128 x 128, resident in shared memory) as B; fp32 accumulator in TMEM, two
-//            128-column buffers so tile i's MMA overlaps tile i-1's epilogue; completion through
-//            tcgen05.commit on an mbarrier (bounded wait).
-//   epilogue warp w reads TMEM lanes 32w..32w+31 (row = slot) 32 columns at a time and stores
-//            coefficient j < r_t of the slot's token at base[r] + j * pad8(n_r) + pos: lanes of
-//            one bucket write consecutive addresses.
+// One CTA owns a range of bucketed slots of one (sequence, layer, head, K-or-V) stream and runs
+// three warp roles over a 5-stage ring of 128-slot tiles:
+//   producers (2 warps)  for tile i: token t = perm[slot]; rank r and in-bucket position p follow
+//                        from the slot alone (tokens sit in slot order inside a bucket: r is found
+//                        by a prefix search over the bucket counts, p = slot - bucket start). Token
+//                        rows (256 B) are gathered with 16-byte cp.async, 16 lanes per row, into a
+//                        128 x 128 bf16 tile in the K-major 128-byte-swizzled layout the tensor core
+//                        reads; once a tile's copies have landed the producers fence the async proxy
+//                        and arrive on the stage's mbarrier (two tiles stay in flight behind it).
+//   mma (1 thread)       8 x tcgen05.mma (M = 128 slots, N = 128 coefficients, K = 16) with U
+//                        (128 x 128, resident in shared memory) as B, into one of two TMEM
+//                        accumulators; tcgen05.commit frees the stage and hands the accumulator on.
+//   epilogue (4 warps)   warp w reads TMEM lanes 32w..32w+31 (row = slot) 32 columns at a time and
+//                        stores coefficient j < r of the slot's token in the tiled bucket layout
+//                        (coef_offset): lanes of one 8-slot group write consecutive addresses.
+// Every mbarrier wait is bounded; a timeout raises VARRATE_ERR_TIMEOUT.
 #include "common.cuh"
 #include "kernels.h"
 
@@ -24,23 +27,27 @@ namespace {
 
 constexpr int kMaxR = kHeadDim;
 constexpr int TM = 128;                    // slots per tile
-constexpr int NST = 5;                     // gather stages
+constexpr int NST = 5;                     // operand stages
+constexpr int NMETA = NST + 2;             // metadata ring (outlives the epilogue of its tile)
+constexpr int LAG = 2;                     // copy groups kept in flight behind the signalled one
 constexpr int TILE_BYTES = TM * kHeadDim * 2;
+constexpr int kEpi = 4, kProd = 2;         // warps
+constexpr int kThreads = (kEpi + kProd + 1) * 32;
 constexpr uint32_t kWaitTries = 1u << 22;  // bounded mbarrier polls
 
 struct ProjSmem {
-  uint64_t mma_bar[2];
+  uint64_t full[NST], empty[NST], tfull[2], tempty[2];
   uint32_t tmem_base;
   int err;
-  int tok[NST][TM];
-  int rk[NST][TM];
-  int ps[NST][TM];
+  int tok[NMETA][TM];
+  int rk[NMETA][TM];
+  int ps[NMETA][TM];
   int n8[kMaxR + 1];
   int slot_start[kMaxR + 2];   // first bucketed slot of rank r (exclusive prefix of the counts)
   long long base[kMaxR + 2];
 };
 
-__global__ void __launch_bounds__(128, 1)
+__global__ void __launch_bounds__(kThreads, 1)
 project_tc_kernel(const __nv_bfloat16* __restrict__ k, const __nv_bfloat16* __restrict__ v,
                   const __nv_bfloat16* __restrict__ basis_k, const __nv_bfloat16* __restrict__ basis_v,
                   const int32_t* __restrict__ bucket_count, const int64_t* __restrict__ bucket_base,
@@ -53,7 +60,7 @@ project_tc_kernel(const __nv_bfloat16* __restrict__ k, const __nv_bfloat16* __re
   unsigned char* stages = smem + TILE_BYTES;                      // NST x 32 KB
   ProjSmem& sm = *reinterpret_cast<ProjSmem*>(stages + NST * TILE_BYTES);
 
-  const int tid = threadIdx.x, warp = tid >> 5;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int64_t bl = blockIdx.z;
   const int g = blockIdx.y >> 1, kv = blockIdx.y & 1;
   const int64_t l = bl % s.L;
@@ -76,18 +83,17 @@ project_tc_kernel(const __nv_bfloat16* __restrict__ k, const __nv_bfloat16* __re
 
   // U of this head into shared memory (row j = basis vector j), swizzled K-major
   const __nv_bfloat16* U = (kv ? basis_v : basis_k) + (l * s.G + g) * (int64_t)kHeadDim * kHeadDim;
-  {
-    const uint4* src = reinterpret_cast<const uint4*>(U + (int64_t)tid * kHeadDim);
-#pragma unroll
-    for (int c = 0; c < 16; ++c)
-      *reinterpret_cast<uint4*>(u_tile + sw128_offset(tid, c, TM)) = __ldg(src + c);
+  for (int idx = tid; idx < TM * 16; idx += blockDim.x) {
+    const int row = idx >> 4, c = idx & 15;
+    *reinterpret_cast<uint4*>(u_tile + sw128_offset(row, c, TM)) =
+        __ldg(reinterpret_cast<const uint4*>(U + (int64_t)row * kHeadDim) + c);
   }
-  if (warp == 0) tmem_alloc(&sm.tmem_base, 256);
-  if (tid == 0) {
-    mbar_init(&sm.mma_bar[0], 1);
-    mbar_init(&sm.mma_bar[1], 1);
+  if (warp == kEpi + kProd && lane == 0) {
+    for (int i = 0; i < NST; ++i) { mbar_init(&sm.full[i], kProd * 32); mbar_init(&sm.empty[i], 1); }
+    for (int i = 0; i < 2; ++i) { mbar_init(&sm.tfull[i], 1); mbar_init(&sm.tempty[i], kEpi); }
     fence_mbar_init();
   }
+  if (warp == 0) tmem_alloc(&sm.tmem_base, 256);
   fence_proxy_async_smem();
   tc_fence_before();
   __syncthreads();
@@ -100,106 +106,127 @@ project_tc_kernel(const __nv_bfloat16* __restrict__ k, const __nv_bfloat16* __re
   const int64_t s_end = min(s.N, s_begin + chunk);
   const int n_tiles = (int)((s_end - s_begin + TM - 1) / TM);
   const uint32_t stage0 = smem_addr(stages), u_addr = smem_addr(u_tile);
-  constexpr uint32_t idesc = idesc_bf16_f32(TM, kHeadDim);
 
-  // perm of the next tile to gather, loaded one iteration ahead (-1 past the range)
-  auto perm_of = [&](int i) -> int {
-    const int64_t slot = s_begin + (int64_t)i * TM + tid;
-    return (i < n_tiles && slot < s_end) ? perm[bl * s.N + slot] : -1;
-  };
-  // slot metadata of row `tid` of tile i (token, rank, position in bucket) into its stage
-  auto stage_meta = [&](int i, int t) {
-    if (i >= n_tiles) return;
-    const int st = i % NST;
-    const int slot = (int)(s_begin + (int64_t)i * TM + tid);
-    int r = 0, p = 0;
-    if (t >= 0) {
-      int lo = 0, hi = kMaxR + 1;   // slot_start[lo] <= slot < slot_start[hi]
-      while (hi - lo > 1) {
-        const int mid = (lo + hi) >> 1;
-        if (sm.slot_start[mid] <= slot) lo = mid; else hi = mid;
+  if (warp >= kEpi && warp < kEpi + kProd) {
+    // ------------------------------------------------------------------ producers
+    const int pt = tid - kEpi * 32;            // 0 .. 63
+    bool bad = false;
+    auto signal = [&](int j) {                 // this thread's copies of tile j have landed
+      fence_proxy_async_smem();
+      mbar_arrive(&sm.full[j % NST]);
+    };
+    // perm of this thread's two rows, one tile ahead of its use
+    auto perm_of = [&](int i, int row) -> int {
+      const int64_t slot = s_begin + (int64_t)i * TM + row;
+      return (i < n_tiles && slot < s_end) ? perm[bl * s.N + slot] : -1;
+    };
+    int t_next[2] = {perm_of(0, pt), perm_of(0, pt + 64)};
+    for (int i = 0; i < n_tiles; ++i) {
+      const int st = i % NST, mt = i % NMETA;
+      const int t_cur[2] = {t_next[0], t_next[1]};
+      t_next[0] = perm_of(i + 1, pt);
+      t_next[1] = perm_of(i + 1, pt + 64);
+      if (!bad && !mbar_wait_bounded(&sm.empty[st], ((i / NST) & 1) ^ 1, kWaitTries)) { sm.err = 1; bad = true; }
+      // bucket of the tile's first slot (same search in every lane: broadcast reads), then a short
+      // forward scan per row: buckets are in slot order
+      const int slot0 = (int)(s_begin + (int64_t)i * TM);
+      int r0 = 0;
+      {
+        int lo = 0, hi = kMaxR + 1;            // slot_start[lo] <= slot0 < slot_start[hi]
+        while (hi - lo > 1) {
+          const int mid = (lo + hi) >> 1;
+          if (sm.slot_start[mid] <= slot0) lo = mid; else hi = mid;
+        }
+        r0 = lo;
       }
-      r = lo;
-      p = slot - sm.slot_start[lo];
-    }
-    sm.tok[st][tid] = t;
-    sm.rk[st][tid] = r;
-    sm.ps[st][tid] = p;
-  };
-  // copies of tile i (after its metadata is visible): 16 lanes per 256-byte row, so one warp
-  // instruction moves two whole rows
-  auto gather = [&](int i) {
-    if (i < n_tiles) {
-      const int st = i % NST;
-      const uint32_t dst = stage0 + st * TILE_BYTES;
-      const int c = tid & 15;
 #pragma unroll
-      for (int q = 0; q < TM / 8; ++q) {
-        const int row = (tid >> 4) + 8 * q;
-        const int t = sm.tok[st][row];
+      for (int h = 0; h < 2; ++h) {
+        const int row = pt + 64 * h;
+        const int slot = slot0 + row;
+        const int t = t_cur[h];
+        int r = 0, p = 0;
+        if (t >= 0) {
+          r = r0;
+          while (sm.slot_start[r + 1] <= slot) ++r;
+          p = slot - sm.slot_start[r];
+        }
+        sm.tok[mt][row] = t;
+        sm.rk[mt][row] = r;
+        sm.ps[mt][row] = p;
+      }
+      named_sync(1, kProd * 32);               // metadata of every row of the tile is visible
+      const uint32_t dst = stage0 + st * TILE_BYTES;
+      const int c = pt & 15;
+#pragma unroll
+      for (int q = 0; q < TM / 4; ++q) {
+        const int row = (pt >> 4) + 4 * q;
+        const int t = sm.tok[mt][row];
         const __nv_bfloat16* src = x + (int64_t)(t < 0 ? 0 : t) * kHeadDim + c * 8;
         cp_async16(dst + sw128_offset(row, c, TM), src, t >= 0 ? 16u : 0u);
       }
+      cp_async_commit();
+      if (i >= LAG) {
+        cp_async_wait<LAG>();
+        signal(i - LAG);
+      }
     }
-    cp_async_commit();
-  };
-
-  auto epilogue = [&](int i) {
-    const bool ok = mbar_wait_bounded(&sm.mma_bar[i & 1], (i >> 1) & 1, kWaitTries);
-    if (!ok) sm.err = 1;
-    tc_fence_after();
-    const int st = i % NST;
-    const int t = sm.tok[st][tid], r = sm.rk[st][tid], p = sm.ps[st][tid];
-    const int rmax_w = __reduce_max_sync(0xffffffffu, t >= 0 ? r : 0);
-    const long long b0 = sm.base[r];
-    const int n8 = sm.n8[r];
-    const uint32_t taddr = tmem + (uint32_t)((i & 1) * kHeadDim) + ((uint32_t)(warp * 32) << 16);
+    cp_async_wait<0>();
+    for (int j = max(0, n_tiles - LAG); j < n_tiles; ++j) signal(j);
+  } else if (warp == kEpi + kProd) {
+    // ------------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t idesc = idesc_bf16_f32(TM, kHeadDim);
+      for (int i = 0; i < n_tiles; ++i) {
+        const int st = i % NST, b = i & 1;
+        if (!mbar_wait_bounded(&sm.full[st], (i / NST) & 1, kWaitTries) ||
+            !mbar_wait_bounded(&sm.tempty[b], ((i >> 1) & 1) ^ 1, kWaitTries)) { sm.err = 1; break; }
+        tc_fence_after();
+        const uint32_t a0 = stage0 + st * TILE_BYTES;
+        const uint32_t d = tmem + (uint32_t)(b * kHeadDim);
 #pragma unroll
-    for (int cb = 0; cb < kHeadDim / 32; ++cb) {
-      if (cb * 32 >= rmax_w) break;            // warp-uniform
-      float vals[32];
-      tmem_ld32(taddr + cb * 32, vals);
-      if (ok && t >= 0) {
+        for (int ks = 0; ks < kHeadDim / 16; ++ks) {
+          const uint32_t off = (ks >> 2) * (TM * 128) + (ks & 3) * 32;
+          tc_mma_bf16(d, sdesc_sw128(a0 + off), sdesc_sw128(u_addr + off), idesc, ks > 0 ? 1u : 0u);
+        }
+        tc_commit(&sm.empty[st]);
+        tc_commit(&sm.tfull[b]);
+      }
+    }
+  } else {
+    // ------------------------------------------------------------------ epilogue
+    bool bad = false;
+    for (int i = 0; i < n_tiles; ++i) {
+      const int b = i & 1, mt = i % NMETA;
+      if (!bad && !mbar_wait_bounded(&sm.tfull[b], (i >> 1) & 1, kWaitTries)) { sm.err = 1; bad = true; }
+      tc_fence_after();
+      const int t = sm.tok[mt][tid], r = sm.rk[mt][tid], p = sm.ps[mt][tid];
+      const int rmax_w = __reduce_max_sync(0xffffffffu, t >= 0 ? r : 0);
+      // this slot's position in its 128-slot tile (coef_offset): the row of coefficient j starts at
+      // tile + j * tl, the slot's 8-group rotates by one position per row
+      const long long p0 = ((long long)p >> 7) << 7;
+      const int tl = (int)min(128LL, (long long)sm.n8[r] - p0);
+      const int ng = max(tl >> 3, 1);
+      const int pl = p - (int)p0;
+      __nv_bfloat16* tile = out + sm.base[r] + p0 * r + (pl & 7);
+      const uint32_t taddr = tmem + (uint32_t)(b * kHeadDim) + ((uint32_t)(warp * 32) << 16);
+      int grp = (pl >> 3) % ng;
+#pragma unroll
+      for (int cb = 0; cb < kHeadDim / 32; ++cb) {
+        if (cb * 32 >= rmax_w) break;          // warp-uniform
+        float vals[32];
+        tmem_ld32(taddr + cb * 32, vals);
 #pragma unroll
         for (int jj = 0; jj < 32; ++jj) {
           const int j = cb * 32 + jj;
-          if (j < r) out[b0 + (long long)j * n8 + p] = __float2bfloat16_rn(vals[jj]);
+          if (!bad && t >= 0 && j < r) tile[(long long)j * tl + grp * 8] = __float2bfloat16_rn(vals[jj]);
+          grp = (grp + 1 == ng) ? 0 : grp + 1;
         }
       }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sm.tempty[b]);
     }
-  };
-
-#pragma unroll
-  for (int i = 0; i < NST - 1; ++i) stage_meta(i, perm_of(i));
-  int t_next = perm_of(NST - 1);
-  __syncthreads();
-#pragma unroll
-  for (int i = 0; i < NST - 1; ++i) gather(i);
-  for (int i = 0; i < n_tiles; ++i) {
-    cp_async_wait<NST - 2>();
-    fence_proxy_async_smem();
-    __syncthreads();
-    if (tid == 0) {
-      tc_fence_after();
-      const uint32_t a0 = stage0 + (i % NST) * TILE_BYTES;
-      const uint32_t d = tmem + (uint32_t)((i & 1) * kHeadDim);
-#pragma unroll
-      for (int ks = 0; ks < kHeadDim / 16; ++ks) {
-        const uint32_t off = (ks >> 2) * (TM * 128) + (ks & 3) * 32;
-        tc_mma_bf16(d, sdesc_sw128(a0 + off), sdesc_sw128(u_addr + off), idesc, ks > 0 ? 1u : 0u);
-      }
-      tc_commit(&sm.mma_bar[i & 1]);
-    }
-    if (i >= 1) epilogue(i - 1);
-    // tile i + NST - 1 reuses the stage of tile i - 1, whose MMA and epilogue are complete
-    stage_meta(i + NST - 1, t_next);
-    t_next = perm_of(i + NST);
-    tc_fence_before();
-    __syncthreads();
-    gather(i + NST - 1);
   }
-  if (n_tiles >= 1) epilogue(n_tiles - 1);
-  cp_async_wait<0>();
   tc_fence_before();
   __syncthreads();
   if (warp == 0) tmem_dealloc(tmem, 256);
@@ -220,7 +247,7 @@ int launch_project_tc(const Shape& s, const void* k, const void* v, const void* 
   const int n_chunks = (int)((s.N + chunk - 1) / chunk);
   const size_t smem = project_tc_smem_bytes();
   cudaFuncSetAttribute(project_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  project_tc_kernel<<<dim3(n_chunks, s.G * 2, s.B * s.L), 128, smem, st>>>(
+  project_tc_kernel<<<dim3(n_chunks, s.G * 2, s.B * s.L), kThreads, smem, st>>>(
       (const __nv_bfloat16*)k, (const __nv_bfloat16*)v, (const __nv_bfloat16*)basis_k,
       (const __nv_bfloat16*)basis_v, out.bucket_count, out.bucket_base, out.perm,
       (__nv_bfloat16*)out.coef, dev_status, s, chunk);

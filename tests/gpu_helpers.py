@@ -70,6 +70,16 @@ def gpu_decode(cfg, packed, bk, bv, q, layer, tail_k=None, tail_v=None):
     return f64(out), int(status.item())
 
 
+def coef_index(base_r, r, n8, p, j):
+    """Element index of coefficient j of bucket slot p in the packed layout of include/varrate.h:
+    128-slot tiles of r rows each, the 8-slot groups of row j rotated by j."""
+    t0 = (p // 128) * 128
+    tl = np.minimum(128, n8 - t0)
+    ng = tl // 8
+    grp = ((p - t0) // 8 + j) % ng
+    return base_r + t0 * r + j * tl + grp * 8 + (p - t0) % 8
+
+
 def unpack(packed, b, l, g, kv, ranks, count, base, pos, d=128):
     """Gather the coefficients of one stream from the device layout using the oracle's tables:
     [N][d] with zeros beyond each token's rank."""
@@ -77,8 +87,9 @@ def unpack(packed, b, l, g, kv, ranks, count, base, pos, d=128):
     ranks = np.asarray(ranks, dtype=np.int64)
     n8 = (np.asarray(count, dtype=np.int64) + 7) // 8 * 8
     j = np.arange(d)[None, :]
-    idx = np.asarray(base)[ranks][:, None] + j * n8[ranks][:, None] + np.asarray(pos)[:, None]
-    mask = j < ranks[:, None]
+    rr = ranks[:, None]
+    idx = coef_index(np.asarray(base)[rr], rr, n8[rr], np.asarray(pos, dtype=np.int64)[:, None], j)
+    mask = j < rr
     out = np.zeros((ranks.size, d))
     out[mask] = buf[idx[mask]]
     return out
