@@ -175,7 +175,10 @@ varrate_status varrate_encode(const varrate_config* cfg, const void* q_win, cons
  *   tail_k/_v [B][G][n_tail][d] uncompressed tokens appended after the cache (may be NULL if
  *           n_tail == 0)
  *   out     [B][H][d]  dtype
- *   ws      at least varrate_workspace_bytes(cfg, VARRATE_CALL_DECODE) bytes. */
+ *   ws      at least varrate_workspace_bytes(cfg, VARRATE_CALL_DECODE) bytes; no contents
+ *           required (in bf16 the call clears its per-(sequence, KV head) completion counters in
+ *           the workspace on `stream` before its one kernel, so calls sharing a workspace must be
+ *           ordered on one stream). */
 varrate_status varrate_decode_attn(const varrate_config* cfg, const varrate_packed* cache,
                                    const void* basis_k, const void* basis_v, const void* q,
                                    int32_t layer, const void* tail_k, const void* tail_v,
@@ -194,7 +197,8 @@ varrate_status varrate_decode_attn(const varrate_config* cfg, const varrate_pack
  *    current device); make that first call before any stream capture.
  *  - All calls share the one array: calls that overlap on the GPU (other streams, other host
  *    threads) race on it and must be serialised by the caller. No contents carry over that matter:
- *    every scratch element is written before it is read. */
+ *    every scratch element is written (the completion counters cleared on the stream) before it
+ *    is read. */
 varrate_status varrate_decode_attn_noalloc(const varrate_config* cfg, const varrate_packed* cache,
                                            const void* basis_k, const void* basis_v, const void* q,
                                            int32_t layer, const void* tail_k, const void* tail_v,

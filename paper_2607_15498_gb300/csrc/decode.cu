@@ -371,7 +371,7 @@ int launch_decode(const Shape& s, const varrate_packed& cache, const void* basis
                   const void* basis_v, const void* q, int layer, const void* tail_k,
                   const void* tail_v, int n_tail, void* out, int32_t* dev_status, void* ws,
                   int num_sms, cudaStream_t st) {
-  if (decode_mma_supported(s, n_tail))
+  if (decode_mma_supported(s, n_tail, num_sms))
     return launch_decode_mma(s, cache, basis_k, basis_v, q, layer, tail_k, tail_v, n_tail, out,
                              dev_status, reinterpret_cast<float*>(ws), num_sms, st);
   const int S = decode_splits(s, num_sms);

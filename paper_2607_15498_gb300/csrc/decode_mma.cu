@@ -24,8 +24,10 @@
 //   softmax  online, per head, 8 heads per tile (grp <= 8; unused heads are computed and ignored)
 //   values   O~^T[j][head] += V[j][slot] * P^T[slot][head]      (P in bf16, <= 2^-9 relative per
 //            weight, transposed from the score fragments with movmatrix)
-// Partials (max, sum, o~[128]) per (segment, CTA) go to the workspace; decode_combine_mma merges
-// them, rotates back with U_V^T (staged in shared memory) and normalises.
+// Partials (max, sum, o~[128]) per (segment, CTA) go to the workspace. The last CTA to finish a
+// segment (a per-segment counter in the workspace, zeroed before the launch) merges its partials,
+// adds the exact tail, rotates back with U_V^T (staged in the idle ring) and normalises, so one
+// launch does the whole step.
 #include <stddef.h>
 
 #include "common.cuh"
@@ -41,10 +43,15 @@ constexpr int ST = 3;                 // ring stages per warp
 constexpr int ISL = 128;              // slots per item
 constexpr int CH = 32;                // coefficient rows per chunk
 constexpr int STAGE = CH * ISL * 2;   // one chunk: up to 32 rows of a 128-slot tile
-constexpr int kPartStride = kHeadDim + 2;
+constexpr int kPartStride = kHeadDim + 4;   // o~[128], max, sum, pad: rows 16-byte aligned
 constexpr int kHeadsPad = 8;
 constexpr uint32_t kWaitTries = 1u << 22;   // bounded mbarrier polls (well over a second)
 constexpr float kSlack = 8.f;                // headroom of the running max, log2 units
+// Cost-line allowance per (sequence, KV head) segment, in K-stream elements: a CTA that enters a
+// segment pays its set-up (tables, query rotation, pipeline ramp, partial write, and for one CTA
+// the combine), about as long as streaming this many coefficients at a CTA's share of HBM
+// bandwidth, so ranges that straddle segments are shortened by that much.
+constexpr long long kSegCost = 98304;
 
 struct SegSmem {
   alignas(16) uint32_t qfrag[kHeadDim / 16][32][4];   // per j-chunk, per lane: b0 hi, b1 hi, b0 lo, b1 lo (read as uint4)
@@ -58,6 +65,8 @@ static_assert(offsetof(SegSmem, qfrag) % 16 == 0, "qfrag is read with 16-byte lo
 
 struct Merge {
   float M[NW][kHeadsPad], L[NW][kHeadsPad];
+  float F[NW][kHeadsPad];             // 2^(M - max): each warp's weight in the CTA's partial
+  float mx[kHeadsPad], l[kHeadsPad];
   float acc[NW][kHeadsPad][kHeadDim];
 };
 
@@ -68,10 +77,17 @@ __device__ __forceinline__ void bucket_range(const SegSmem& sm, int r, long long
                                              long long& i0, long long& i1) {
   const int n = sm.cnt[r];
   if (n == 0) { i0 = i1 = 0; return; }
-  const long long n8 = pad8(n), b0 = sm.base[r], unit = (long long)ISL * r;
+  const long long n8 = pad8(n), b0 = sm.base[r];
   const long long nit = (n8 + ISL - 1) / ISL;
-  i0 = lo > b0 ? (lo - b0 + unit - 1) / unit : 0;
-  i1 = hi > b0 ? (hi - b0 + unit - 1) / unit : 0;
+  // ceil(x / (128 r)) = ceil(ceil(x / 128) / r)
+  auto items_before = [&](long long x) -> long long {
+    if (x <= 0) return 0;
+    const unsigned long long a = ((unsigned long long)x + ISL - 1) / ISL;
+    if (a < (1ull << 31)) return (long long)(((uint32_t)a + (uint32_t)r - 1u) / (uint32_t)r);
+    return (long long)((a + r - 1) / r);
+  };
+  i0 = items_before(lo - b0);
+  i1 = items_before(hi - b0);
   if (i1 > nit) i1 = nit;
   if (i0 > i1) i0 = i1;
 }
@@ -119,7 +135,8 @@ __device__ __forceinline__ bool issue_chunk(Prod& p, const SegSmem& sm, const __
     const uint32_t bytes = (uint32_t)(rows * tl * 2);           // rows j0.. of the tile: contiguous
     mbar_arrive_expect_tx(bar, bytes);
     fence_proxy_async_smem();  // the generic reads above precede the async write
-    bulk_g2s(stage_addr, (p.phase ? cV : cK) + sm.base[r] + t0 * r + (long long)j0 * tl, bytes, bar);
+    bulk_g2s_hint(stage_addr, (p.phase ? cV : cK) + sm.base[r] + t0 * r + (long long)j0 * tl, bytes, bar,
+                  l2_evict_first_policy());
   }
   const int nj = (r + CH - 1) / CH;
   if (++p.jc == nj) {
@@ -148,37 +165,46 @@ __device__ __forceinline__ uint32_t keep_rows(uint32_t w, int j, int r) {
 }
 
 // Rotate the queries of (b, g) into the basis: qt[head][j] = scale * sum_i U_K[j][i] q[head][i],
-// warp w computing rows j in [16w, 16w + 16) with one m16n8k16 tile per 16 columns of U_K.
-__device__ void rotate_queries(SegSmem& sm, const __nv_bfloat16* __restrict__ U,
-                               const __nv_bfloat16* __restrict__ q, int grp, int warp, int lane) {
-  const int g8 = lane >> 2, c = lane & 3;
-  const float scale = kLog2e * rsqrtf((float)kHeadDim);
-  for (int mt = warp; mt < kHeadDim / 16; mt += NW) {
-    float d[4] = {0.f, 0.f, 0.f, 0.f};
-    const int j0 = mt * 16;
+// warp w computing rows j in [16w, 16w + 16) with one m16n8k16 tile per 16 columns of U_K. The
+// loads (rot_load) are issued at the start of a segment, ahead of its table loads, so both take
+// one memory round trip together; rot_compute runs once the tables are in.
+static_assert(NW * 16 == kHeadDim, "one 16-row tile of U_K per warp");
+struct RotRegs {
+  uint32_t a[kHeadDim / 16][4];    // U_K rows 16w .. 16w + 15 (A fragments)
+  uint32_t bq[kHeadDim / 16][2];   // q (B fragments; zero for padded heads)
+};
+
+__device__ __forceinline__ void rot_load(RotRegs& rr, const __nv_bfloat16* __restrict__ U,
+                                         const __nv_bfloat16* __restrict__ q, int grp, int warp, int lane) {
+  const int g8 = lane >> 2, c = lane & 3, j0 = warp * 16;
+  const uint32_t* Uw = reinterpret_cast<const uint32_t*>(U);
+  const uint32_t* qw = reinterpret_cast<const uint32_t*>(q + (long long)(g8 < grp ? g8 : 0) * kHeadDim);
 #pragma unroll
-    for (int kc = 0; kc < kHeadDim / 16; ++kc) {
-      const int i0 = kc * 16;
-      uint32_t a[4];
-      const uint32_t* Uw = reinterpret_cast<const uint32_t*>(U);
-      a[0] = __ldg(Uw + ((j0 + g8) * kHeadDim + i0 + 2 * c) / 2);
-      a[1] = __ldg(Uw + ((j0 + g8 + 8) * kHeadDim + i0 + 2 * c) / 2);
-      a[2] = __ldg(Uw + ((j0 + g8) * kHeadDim + i0 + 2 * c + 8) / 2);
-      a[3] = __ldg(Uw + ((j0 + g8 + 8) * kHeadDim + i0 + 2 * c + 8) / 2);
-      uint32_t b0 = 0, b1 = 0;
-      if (g8 < grp) {
-        const uint32_t* qw = reinterpret_cast<const uint32_t*>(q + (long long)g8 * kHeadDim);
-        b0 = __ldg(qw + (i0 + 2 * c) / 2);
-        b1 = __ldg(qw + (i0 + 2 * c + 8) / 2);
-      }
-      mma_bf16_16816(d, a, b0, b1);
-    }
-    // d: rows j0+g8 (+8), heads 2c, 2c+1
-    sm.qt[2 * c][j0 + g8] = d[0] * scale;
-    sm.qt[2 * c + 1][j0 + g8] = d[1] * scale;
-    sm.qt[2 * c][j0 + g8 + 8] = d[2] * scale;
-    sm.qt[2 * c + 1][j0 + g8 + 8] = d[3] * scale;
+  for (int kc = 0; kc < kHeadDim / 16; ++kc) {
+    const int i0 = kc * 16;
+    rr.a[kc][0] = __ldg(Uw + ((j0 + g8) * kHeadDim + i0 + 2 * c) / 2);
+    rr.a[kc][1] = __ldg(Uw + ((j0 + g8 + 8) * kHeadDim + i0 + 2 * c) / 2);
+    rr.a[kc][2] = __ldg(Uw + ((j0 + g8) * kHeadDim + i0 + 2 * c + 8) / 2);
+    rr.a[kc][3] = __ldg(Uw + ((j0 + g8 + 8) * kHeadDim + i0 + 2 * c + 8) / 2);
+    rr.bq[kc][0] = __ldg(qw + (i0 + 2 * c) / 2);
+    rr.bq[kc][1] = __ldg(qw + (i0 + 2 * c + 8) / 2);
   }
+}
+
+__device__ __forceinline__ void rot_compute(SegSmem& sm, const RotRegs& rr, int grp, int warp, int lane) {
+  const int g8 = lane >> 2, c = lane & 3, j0 = warp * 16;
+  const float scale = kLog2e * rsqrtf((float)kHeadDim);
+  float d[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+  for (int kc = 0; kc < kHeadDim / 16; ++kc) {
+    const uint32_t b0 = g8 < grp ? rr.bq[kc][0] : 0u, b1 = g8 < grp ? rr.bq[kc][1] : 0u;
+    mma_bf16_16816(d, rr.a[kc], b0, b1);
+  }
+  // d: rows j0+g8 (+8), heads 2c, 2c+1
+  sm.qt[2 * c][j0 + g8] = d[0] * scale;
+  sm.qt[2 * c + 1][j0 + g8] = d[1] * scale;
+  sm.qt[2 * c][j0 + g8 + 8] = d[2] * scale;
+  sm.qt[2 * c + 1][j0 + g8 + 8] = d[3] * scale;
 }
 
 // Score-MMA B fragments of q~ (split hi + lo) for every 16-row chunk, one uint4 per lane.
@@ -196,21 +222,179 @@ __device__ void build_qfrag(SegSmem& sm, int tid) {
   }
 }
 
+// Start of CTA c's range on a cost line of T elements cut into C equal ranges: floor(T c / C).
+// The launcher guarantees T * C < 2^63.
+__device__ __forceinline__ long long cut_at(long long T, long long c, int C) {
+  return (long long)(((unsigned long long)T * (unsigned long long)c) / (unsigned long long)C);
+}
+
+// CTAs whose cost range [cuts[c], cuts[c + 1]) meets [P, P + W): c0..c1 (W > 0).
+__device__ __forceinline__ void seg_cta_range(const long long* cuts, int C, long long P, long long W,
+                                              int& c0, int& c1) {
+  int lo = 0, hi = C - 1;   // first c with cuts[c + 1] > P (cuts[C] = T > P)
+  while (lo < hi) {
+    const int mid = (lo + hi) >> 1;
+    if (cuts[mid + 1] > P) hi = mid; else lo = mid + 1;
+  }
+  c0 = lo;
+  lo = c0; hi = C;          // first c with cuts[c] > P + W - 1, or C
+  while (lo < hi) {
+    const int mid = (lo + hi) >> 1;
+    if (cuts[mid] > P + W - 1) hi = mid; else lo = mid + 1;
+  }
+  c1 = lo - 1;
+}
+
+constexpr int kMaxCtas = 1024;   // grid size bound (64-bit cost-line arithmetic)
+
+struct CombSmem {   // aliases the ring while the last CTA of a segment combines it
+  alignas(128) __nv_bfloat16 us[kHeadDim * kHeadDim];   // U_V[g], row j (one bulk copy)
+  float ot[kHeadsPad][kHeadDim + 8];                    // merged o~ per head
+  float qrow[kHeadsPad][kHeadDim];
+  float tsc[kHeadsPad][64];                             // exact tail scores, then weights (n_tail <= 64)
+  float tmax[kHeadsPad], hl[kHeadsPad];
+};
+static_assert(sizeof(CombSmem) <= (size_t)NW * ST * STAGE, "combine buffers fit in the ring");
+static_assert(NW == kHeadsPad, "one warp per head in the combine");
+
+// Merge the partials of segment (b, g) written by CTAs c0..c1 (slot cc + seg; none if c1 < c0),
+// add the exact tail, rotate back with U_V^T (m16n8k16 tiles, o~ split hi + lo) and normalise.
+// Called by all 256 threads; the ring is idle. Warp h merges head h, lane l columns 4l .. 4l + 3,
+// with the partials of up to 8 CTAs in flight at once (online rescaling across batches).
+// Returns false if the U_V copy timed out.
+__device__ bool combine_segment(CombSmem& cs, uint64_t* bar, uint32_t parity, const float* __restrict__ part,
+                                int c0, int c1, long long seg, const __nv_bfloat16* __restrict__ q,
+                                const __nv_bfloat16* __restrict__ Uv, const __nv_bfloat16* __restrict__ tail_k,
+                                const __nv_bfloat16* __restrict__ tail_v, int n_tail,
+                                __nv_bfloat16* __restrict__ out, int grp, int tid) {
+  const int lane = tid & 31, warp = tid >> 5;
+  const int g8 = lane >> 2, c = lane & 3;
+  fence_proxy_async_smem();   // earlier generic accesses of the ring precede the async write
+  __syncthreads();
+  if (tid == 0) {
+    mbar_arrive_expect_tx(bar, kHeadDim * kHeadDim * 2);
+    bulk_g2s(smem_addr(cs.us), Uv, kHeadDim * kHeadDim * 2, bar);
+  }
+  const float scale = kLog2e * rsqrtf((float)kHeadDim);
+  if (n_tail) {                                                   // exact tail scores and maxima
+    for (int i = tid; i < grp * kHeadDim; i += blockDim.x) cs.qrow[i / kHeadDim][i % kHeadDim] = __bfloat162float(q[i]);
+    __syncthreads();
+    for (int i = warp; i < grp * n_tail; i += NW) {
+      const int h = i / n_tail, t = i % n_tail;
+      const __nv_bfloat16* tk = tail_k + (long long)t * kHeadDim;
+      float a = 0.f;
+#pragma unroll
+      for (int k = 0; k < 4; ++k) a = fmaf(cs.qrow[h][lane * 4 + k], __bfloat162float(tk[lane * 4 + k]), a);
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) a += __shfl_xor_sync(0xffffffffu, a, o);
+      if (lane == 0) cs.tsc[h][t] = a * scale;
+    }
+    __syncthreads();
+  }
+  const int h = warp;
+  float M = -INFINITY, L = 0.f;
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (h < grp) {
+    for (int t = lane; t < n_tail; t += 32) M = fmaxf(M, cs.tsc[h][t]);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+    const int np = c1 - c0 + 1;
+    for (int cb = 0; cb < np; cb += 8) {
+      float m[8], l[8];
+      float4 o[8];
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        if (cb + k < np) {
+          const float* pp = part + ((c0 + cb + k + seg) * kHeadsPad + h) * kPartStride;
+          m[k] = __ldcg(pp + kHeadDim);
+          l[k] = __ldcg(pp + kHeadDim + 1);
+          o[k] = __ldcg(reinterpret_cast<const float4*>(pp) + lane);
+        } else {
+          m[k] = -INFINITY; l[k] = 0.f; o[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+      }
+      float mx = M;
+#pragma unroll
+      for (int k = 0; k < 8; ++k) mx = fmaxf(mx, m[k]);
+      if (mx != -INFINITY) {
+        const float f = M == -INFINITY ? 0.f : exp2f(M - mx);
+        acc.x *= f; acc.y *= f; acc.z *= f; acc.w *= f;
+        L *= f;
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+          const float w = m[k] == -INFINITY ? 0.f : exp2f(m[k] - mx);
+          L = fmaf(w, l[k], L);
+          acc.x = fmaf(w, o[k].x, acc.x); acc.y = fmaf(w, o[k].y, acc.y);
+          acc.z = fmaf(w, o[k].z, acc.z); acc.w = fmaf(w, o[k].w, acc.w);
+        }
+        M = mx;
+      }
+    }
+    float lt = 0.f;                                               // tail weights at the final max
+    for (int t = lane; t < n_tail; t += 32) {
+      const float w = exp2f(cs.tsc[h][t] - M);
+      cs.tsc[h][t] = w;
+      lt += w;
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) lt += __shfl_xor_sync(0xffffffffu, lt, o);
+    if (lane == 0) cs.hl[h] = L + lt;
+  }
+  *reinterpret_cast<float4*>(&cs.ot[h][4 * lane]) = acc;        // zero for padded heads
+  if (!__syncthreads_and(mbar_wait_bounded(bar, parity, kWaitTries))) return false;
+  // out^T[col][head] = sum_j U_V[j][col] o~[head][j]: warp w owns columns 16w .. 16w + 15
+  {
+    float d[4] = {0.f, 0.f, 0.f, 0.f};
+    const int col0 = warp * 16;
+#pragma unroll
+    for (int ks = 0; ks < kHeadDim / 16; ++ks) {
+      const int j = ks * 16 + (lane & 7) + ((lane >> 4) & 1) * 8;
+      const int col = col0 + ((lane >> 3) & 1) * 8;
+      uint32_t a[4];
+      ldsm_x4_trans(smem_addr(&cs.us[j * kHeadDim + col]), a);
+      const int jb = ks * 16 + 2 * c;
+      uint32_t h0, l0, h1, l1;
+      split_bf16(cs.ot[g8][jb], cs.ot[g8][jb + 1], h0, l0);
+      split_bf16(cs.ot[g8][jb + 8], cs.ot[g8][jb + 9], h1, l1);
+      mma_bf16_16816(d, a, h0, h1);
+      mma_bf16_16816(d, a, l0, l1);
+    }
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const int col = col0 + g8 + (e >> 1) * 8, hh = 2 * c + (e & 1);
+      if (hh < grp) {
+        float y = d[e];
+        for (int t = 0; t < n_tail; ++t)
+          y = fmaf(cs.tsc[hh][t], __bfloat162float(tail_v[(long long)t * kHeadDim + col]), y);
+        out[(long long)hh * kHeadDim + col] = __float2bfloat16_rn(y / cs.hl[hh]);
+      }
+    }
+  }
+  return true;
+}
+
 __global__ void __launch_bounds__(NW * 32, 1)
 decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restrict__ bucket_count,
                   const int64_t* __restrict__ bucket_base, const __nv_bfloat16* __restrict__ basis_k,
-                  const __nv_bfloat16* __restrict__ qin, float* __restrict__ part,
-                  int32_t* __restrict__ dev_status, Shape s, int layer) {
+                  const __nv_bfloat16* __restrict__ basis_v, const __nv_bfloat16* __restrict__ qin,
+                  const __nv_bfloat16* __restrict__ tail_k, const __nv_bfloat16* __restrict__ tail_v,
+                  int n_tail, __nv_bfloat16* __restrict__ out, float* __restrict__ part,
+                  int* __restrict__ seg_done, int32_t* __restrict__ dev_status, Shape s, int layer) {
   extern __shared__ __align__(128) unsigned char smem[];
   unsigned char* ring = smem;                                     // NW * ST * STAGE
   static_assert((NW * ST * STAGE) % 16 == 0, "SegSmem must start 16-byte aligned");
   SegSmem& sm = *reinterpret_cast<SegSmem*>(smem + NW * ST * STAGE);
-  // the merge buffers alias the ring; the ring is zeroed again after every merge so that it only
-  // ever holds finite coefficients or zeros
+  // the merge and combine buffers alias the ring; the ring is zeroed again after every merge so
+  // that it only ever holds finite coefficients or zeros
   static_assert(sizeof(Merge) <= (size_t)NW * ST * STAGE, "merge buffers fit in the ring");
   Merge& mg = *reinterpret_cast<Merge*>(smem);
   __shared__ long long segW[64];                                  // per-sequence stream length
+  __shared__ long long segP[65];                                  // start of sequence b on the cost line
+  __shared__ long long cuts[kMaxCtas + 1];                        // start of CTA c's range
+  __shared__ int n_empty;                                         // sequences with no coded tokens
+  __shared__ int last_cta;                                        // this CTA closes the segment
   __shared__ uint64_t bar_all[NW * ST];                           // one full-barrier per ring stage
+  __shared__ uint64_t bar_comb;                                   // U_V copy of a combine
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int g8 = lane >> 2, c = lane & 3;
@@ -221,6 +405,7 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
   for (int i = tid; i < NW * ST * STAGE / 16; i += blockDim.x)
     reinterpret_cast<uint4*>(ring)[i] = make_uint4(0, 0, 0, 0);
   if (tid < NW * ST) mbar_init(&bar_all[tid], 1);
+  if (tid == NW * ST) mbar_init(&bar_comb, 1);
   fence_mbar_init();
   fence_proxy_async_smem();
   pdl_wait();   // everything below reads data written by earlier grids
@@ -233,19 +418,56 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
   uint32_t n_issued = 0;   // chunks this warp has consumed (== index of its next chunk)
   int n_pending = 0;       // chunks issued but not yet consumed
   bool timed_out = false;
-  long long T = 0;
-  for (int b = 0; b < s.B; ++b) T += segW[b] * s.G;
-  if (T == 0) { pdl_trigger(); return; }
-  const long long lo_g = (long long)((__int128)T * cta / C);
-  const long long hi_g = (long long)((__int128)T * (cta + 1) / C);
+  uint32_t n_comb = 0;     // combines done by this CTA (phase of bar_comb)
+  // Cost line: sequence b holds G segments of kSegCost + W_b elements each (W_b > 0), the set-up
+  // allowance first. segP = exclusive prefix over sequences (B <= 64: two per lane).
+  if (warp == 0) {
+    const int e0 = 2 * lane, e1 = 2 * lane + 1;
+    const long long v0 = (e0 < s.B && segW[e0]) ? (segW[e0] + kSegCost) * s.G : 0;
+    const long long v1 = (e1 < s.B && segW[e1]) ? (segW[e1] + kSegCost) * s.G : 0;
+    long long inc = v0 + v1;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const long long y = __shfl_up_sync(0xffffffffu, inc, o);
+      if (lane >= o) inc += y;
+    }
+    segP[e0] = inc - v0 - v1;
+    segP[e1] = inc - v1;
+    if (lane == 31) segP[64] = inc;
+    const unsigned m0 = __ballot_sync(0xffffffffu, e0 < s.B && segW[e0] == 0);
+    const unsigned m1 = __ballot_sync(0xffffffffu, e1 < s.B && segW[e1] == 0);
+    if (lane == 0) n_empty = __popc(m0) + __popc(m1);
+  }
+  __syncthreads();
+  const long long T = segP[64];
+  for (int c2 = tid; c2 <= C; c2 += blockDim.x) cuts[c2] = cut_at(T, c2, C);
+  __syncthreads();
+  const long long lo_g = cuts[cta], hi_g = cuts[cta + 1];
 
-  long long P = 0;   // start of segment (b, g) on the cost line
-  for (int b = 0; b < s.B; ++b) {
-    const long long W = segW[b];
-    for (int g = 0; g < s.G; ++g, P += W) {
-      if (W == 0 || P + W <= lo_g || P >= hi_g) continue;
+  // first segment of this CTA: the sequence whose span holds lo_g, then the head within it
+  int b = 0, g = 0;
+  {
+    int lo_b = 0, hi_b = s.B;
+    while (lo_b < hi_b) {
+      const int mid = (lo_b + hi_b) >> 1;
+      if (segP[mid + 1] > lo_g) hi_b = mid; else lo_b = mid + 1;
+    }
+    b = lo_b;
+    if (b < s.B) g = (int)((lo_g - segP[b]) / (segW[b] + kSegCost));
+  }
+  auto seg_start = [&](int bb, int gg) { return segP[bb] + gg * (segW[bb] + kSegCost) + kSegCost; };
+  bool more = b < s.B && seg_start(b, g) < hi_g;
+  while (more) {
+    {
+      const long long W = segW[b];
+      const long long P = seg_start(b, g);   // first coefficient of segment (b, g) on the cost line
       const long long lo = max(lo_g, P) - P, hi = min(hi_g, P + W) - P;
       const long long bl = (long long)b * s.L + layer;
+      RotRegs rr;   // this segment's U_K tile and queries, in flight with the table loads below
+      rot_load(rr, basis_k + ((long long)layer * s.G + g) * kHeadDim * kHeadDim,
+               qin + ((long long)b * s.H + (long long)g * s.grp) * kHeadDim, s.grp, warp, lane);
+      // U_V of this head, for whichever CTA merges the segment: into L2 while it streams
+      if (tid == 0) bulk_prefetch_l2(basis_v + ((long long)layer * s.G + g) * kHeadDim * kHeadDim, kHeadDim * kHeadDim * 2);
       __syncthreads();
       for (int r = tid; r <= kMaxR + 1; r += blockDim.x) {
         if (r <= kMaxR) sm.cnt[r] = bucket_count[bl * (kMaxR + 1) + r];
@@ -259,10 +481,28 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
         sm.it_pref[r + 1] = (int)(i1 - i0);   // counts first, prefixed below
       }
       __syncthreads();
-      if (tid == 0) {
-        int acc = 0;
-        sm.it_pref[0] = 0;
-        for (int r = 0; r <= kMaxR; ++r) { acc += sm.it_pref[r + 1]; sm.it_pref[r + 1] = acc; }
+      if (warp == 0) {   // inclusive scan of it_pref[1 .. 129], 5 entries per lane
+        constexpr int kPer = (kMaxR + 1 + 31) / 32;
+        int v[kPer], acc = 0;
+#pragma unroll
+        for (int e = 0; e < kPer; ++e) {
+          const int r = lane * kPer + e;
+          acc += r <= kMaxR ? sm.it_pref[r + 1] : 0;
+          v[e] = acc;
+        }
+        int excl = acc;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const int y = __shfl_up_sync(0xffffffffu, excl, o);
+          if (lane >= o) excl += y;
+        }
+        excl -= acc;
+#pragma unroll
+        for (int e = 0; e < kPer; ++e) {
+          const int r = lane * kPer + e;
+          if (r <= kMaxR) sm.it_pref[r + 1] = excl + v[e];
+        }
+        if (lane == 0) sm.it_pref[0] = 0;
       }
       __syncthreads();
       // start this warp's loads first: they do not depend on the rotated queries
@@ -286,8 +526,9 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
       for (int i = 0; i < ST - 1; ++i)
         if (issue_chunk(pr, sm, cK, cV, ring_w + ((n_issued + i) % ST) * STAGE,
                         &bars[(n_issued + i) % ST], total, lane)) ++n_pending;
-      rotate_queries(sm, basis_k + ((long long)layer * s.G + g) * kHeadDim * kHeadDim,
-                     qin + ((long long)b * s.H + (long long)g * s.grp) * kHeadDim, s.grp, warp, lane);
+      int c0, c1;   // the CTAs that share this segment (their partials are merged by the last one)
+      seg_cta_range(cuts, C, P, W, c0, c1);
+      rot_compute(sm, rr, s.grp, warp, lane);
       __syncthreads();
       build_qfrag(sm, tid);
       __syncthreads();
@@ -315,6 +556,7 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
         // stored at position (g + j) mod (tl / 8)
         const int tl = (int)min((long long)ISL, pad8(sm.cnt[r]) - (long long)cons.it * ISL);
         const int ng = tl >> 3;
+        const bool full_tile = ng == 16;
         const uint32_t row_bytes = (uint32_t)tl * 2u;
         float sc[ISL / 16][4];
 #pragma unroll
@@ -330,15 +572,17 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
             const int j16 = jc * CH + ks * 16;
             if (j16 >= r) break;                        // warp-uniform
             uint4 qf = *reinterpret_cast<const uint4*>(&sm.qfrag[j16 >> 4][lane][0]);
-            const int jb = j16 + 2 * c;
-            qf.x = keep_rows(qf.x, jb, r); qf.z = keep_rows(qf.z, jb, r);
-            qf.y = keep_rows(qf.y, jb + 8, r); qf.w = keep_rows(qf.w, jb + 8, r);
+            if (j16 + 16 > r) {                          // warp-uniform: rows >= r in this k-step
+              const int jb = j16 + 2 * c;
+              qf.x = keep_rows(qf.x, jb, r); qf.z = keep_rows(qf.z, jb, r);
+              qf.y = keep_rows(qf.y, jb + 8, r); qf.w = keep_rows(qf.w, jb + 8, r);
+            }
             // this lane's row of the 8x8 matrices: coefficient j, staged at row (j - chunk start)
             const int jrow = ks * 16 + (m >> 1) * 8 + r8;
             const int j = jc * CH + jrow;
             const uint32_t row_addr = st_addr + jrow * row_bytes;
             uint32_t a[ISL / 16][4];
-            int pg = ((m & 1) + j) % ng;                // stored position of slot group 2 mt + (m & 1)
+            int pg = full_tile ? (((m & 1) + j) & 15) : (((m & 1) + j) % ng);   // slot group 2 mt + (m & 1)
 #pragma unroll
             for (int mt = 0; mt < ISL / 16; ++mt) {
               ldsm_x4_trans(row_addr + 16 * pg, a[mt]);
@@ -419,7 +663,7 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
             const uint32_t row_addr = st_addr + jrow * row_bytes;
             const bool keep0 = jt * 16 + g8 < r, keep1 = jt * 16 + g8 + 8 < r;
             float t1[4] = {0.f, 0.f, 0.f, 0.f};
-            int pg = ((m >> 1) + j) % ng;               // stored position of slot group 2 kt + (m >> 1)
+            int pg = full_tile ? (((m >> 1) + j) & 15) : (((m >> 1) + j) % ng);  // slot group 2 kt + (m >> 1)
 #pragma unroll
             for (int kt = 0; kt < ISL / 16; kt += 2) {
               uint32_t a[4], b[4];
@@ -427,8 +671,10 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
               pg = wrap2(pg, ng);
               ldsm_x4(row_addr + 16 * pg, b);
               pg = wrap2(pg, ng);
-              if (!keep0) { a[0] = a[2] = 0u; b[0] = b[2] = 0u; }
-              if (!keep1) { a[1] = a[3] = 0u; b[1] = b[3] = 0u; }
+              if (jt * 16 + 16 > r) {                    // warp-uniform: rows >= r in this tile
+                if (!keep0) { a[0] = a[2] = 0u; b[0] = b[2] = 0u; }
+                if (!keep1) { a[1] = a[3] = 0u; b[1] = b[3] = 0u; }
+              }
               mma_bf16_16816(oacc[jt], a, pb[kt][0], pb[kt][1]);
               mma_bf16_16816(t1, b, pb[kt + 1][0], pb[kt + 1][1]);
             }
@@ -465,136 +711,80 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
         mg.acc[warp][2 * c][t * 16 + g8 + 8] = oacc[t][2];
         mg.acc[warp][2 * c + 1][t * 16 + g8 + 8] = oacc[t][3];
       }
-      __syncthreads();
-      // partial slot of this (segment, CTA): index cta + segment number (unique, see combine)
-      const long long seg = (long long)b * s.G + g;
-      float* out = part + (cta + seg) * (long long)kHeadsPad * kPartStride;
-      for (int i = tid; i < kHeadsPad * kHeadDim; i += blockDim.x) {
-        const int h = i / kHeadDim, j = i % kHeadDim;
-        float mx = -INFINITY;
+      if (tid < kHeadsPad) {
+        const int h = tid;
+        float mx = -INFINITY, l = 0.f;
 #pragma unroll
         for (int w = 0; w < NW; ++w) mx = fmaxf(mx, mg.M[w][h]);
-        float o = 0.f, l = 0.f;
-        if (mx != -INFINITY) {
 #pragma unroll
-          for (int w = 0; w < NW; ++w) {
-            const float f = fast_exp2(mg.M[w][h] - mx);
-            o = fmaf(mg.acc[w][h][j], f, o);
-            l = fmaf(mg.L[w][h], f, l);
-          }
+        for (int w = 0; w < NW; ++w) {
+          const float f = mx == -INFINITY ? 0.f : fast_exp2(mg.M[w][h] - mx);
+          mg.F[w][h] = f;
+          l = fmaf(mg.L[w][h], f, l);
         }
-        out[h * kPartStride + j] = o;
-        if (j == 0) { out[h * kPartStride + kHeadDim] = mx; out[h * kPartStride + kHeadDim + 1] = l; }
+        mg.mx[h] = mx;
+        mg.l[h] = l;
       }
       __syncthreads();
+      // partial slot of this (segment, CTA): index cta + segment number (unique: a CTA after this
+      // one only meets segments after this one)
+      const long long seg = (long long)b * s.G + g;
+      float* pout = part + (cta + seg) * (long long)kHeadsPad * kPartStride;
+      for (int i = tid; i < kHeadsPad * kHeadDim; i += blockDim.x) {
+        const int h = i / kHeadDim, j = i % kHeadDim;
+        float o = 0.f;
+#pragma unroll
+        for (int w = 0; w < NW; ++w) o = fmaf(mg.acc[w][h][j], mg.F[w][h], o);
+        pout[h * kPartStride + j] = o;
+        if (j == 0) { pout[h * kPartStride + kHeadDim] = mg.mx[h]; pout[h * kPartStride + kHeadDim + 1] = mg.l[h]; }
+      }
+      // the last CTA to finish this segment merges every partial of it
+      __syncthreads();
+      if (tid == 0) {
+        __threadfence();
+        last_cta = atomicAdd(&seg_done[seg], 1) == c1 - c0;
+      }
+      __syncthreads();
+      if (last_cta) {
+        __threadfence();
+        if (!combine_segment(*reinterpret_cast<CombSmem*>(ring), &bar_comb, n_comb & 1u, part, c0, c1, seg,
+                             qin + ((long long)b * s.H + (long long)g * s.grp) * kHeadDim,
+                             basis_v + ((long long)layer * s.G + g) * kHeadDim * kHeadDim,
+                             n_tail ? tail_k + ((long long)b * s.G + g) * n_tail * kHeadDim : nullptr,
+                             n_tail ? tail_v + ((long long)b * s.G + g) * n_tail * kHeadDim : nullptr, n_tail,
+                             out + ((long long)b * s.H + (long long)g * s.grp) * kHeadDim, s.grp, tid))
+          timed_out = true;
+        ++n_comb;
+      }
+      __syncthreads();
+    }
+    if (++g == s.G) { ++b; g = 0; }
+    while (b < s.B && segW[b] == 0) ++b;
+    more = b < s.B && seg_start(b, g) < hi_g;
+    if (more) {
       for (int i = tid; i < NW * ST * STAGE / 16; i += blockDim.x)
         reinterpret_cast<uint4*>(ring)[i] = make_uint4(0, 0, 0, 0);
       fence_proxy_async_smem();
       __syncthreads();
     }
   }
+  // segments with an empty coded stream (tail only): one CTA each, no partials
+  if (n_empty)
+  for (int b = 0; b < s.B; ++b)
+    for (int g = 0; g < s.G; ++g) {
+      const long long seg = (long long)b * s.G + g;
+      if (segW[b] != 0 || seg % C != cta) continue;   // CTA-uniform
+      __syncthreads();
+      if (!combine_segment(*reinterpret_cast<CombSmem*>(ring), &bar_comb, n_comb & 1u, part, 0, -1, seg,
+                           qin + ((long long)b * s.H + (long long)g * s.grp) * kHeadDim,
+                           basis_v + ((long long)layer * s.G + g) * kHeadDim * kHeadDim,
+                           n_tail ? tail_k + ((long long)b * s.G + g) * n_tail * kHeadDim : nullptr,
+                           n_tail ? tail_v + ((long long)b * s.G + g) * n_tail * kHeadDim : nullptr, n_tail,
+                           out + ((long long)b * s.H + (long long)g * s.grp) * kHeadDim, s.grp, tid))
+        timed_out = true;
+      ++n_comb;
+    }
   if (timed_out && lane == 0) raise_status(dev_status, VARRATE_ERR_TIMEOUT);
-  pdl_trigger();
-}
-
-// grid (G, B), 256 threads: merge the partials of segment (b, g), add the exact tail, rotate back.
-__global__ void __launch_bounds__(256)
-decode_combine_mma_kernel(const float* __restrict__ part, const int64_t* __restrict__ bucket_base,
-                          const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __restrict__ basis_v,
-                          const __nv_bfloat16* __restrict__ tail_k, const __nv_bfloat16* __restrict__ tail_v,
-                          int n_tail, __nv_bfloat16* __restrict__ out, Shape s, int layer, int C) {
-  __shared__ __align__(16) __nv_bfloat16 us[kHeadDim * kHeadDim];   // U_V[g], row j
-  __shared__ float ot[kHeadsPad][kHeadDim];
-  __shared__ float qrow[kHeadsPad][kHeadDim];
-  __shared__ float tsc[kHeadsPad][64];
-  __shared__ float hm[kHeadsPad], hl[kHeadsPad];
-  __shared__ long long segW[64];
-  const int g = blockIdx.x, b = blockIdx.y;
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-
-  const uint4* src = reinterpret_cast<const uint4*>(basis_v + ((long long)layer * s.G + g) * kHeadDim * kHeadDim);
-  for (int i = tid; i < kHeadDim * kHeadDim / 8; i += blockDim.x) reinterpret_cast<uint4*>(us)[i] = src[i];
-  for (int bb = tid; bb < s.B; bb += blockDim.x) {
-    const long long w = bucket_base[((long long)bb * s.L + layer) * (kMaxR + 2) + kMaxR + 1];
-    segW[bb] = (w >= 0 && w <= s.cap) ? w : 0;
-  }
-  for (int i = tid; i < s.grp * kHeadDim; i += blockDim.x)
-    qrow[i / kHeadDim][i % kHeadDim] =
-        __bfloat162float(q[((long long)b * s.H + (long long)g * s.grp) * kHeadDim + i]);
-  __syncthreads();
-  long long T = 0, P = 0;
-  for (int bb = 0; bb < s.B; ++bb) T += segW[bb] * s.G;
-  for (int bb = 0; bb < b; ++bb) P += segW[bb] * s.G;
-  const long long W = segW[b];
-  P += (long long)g * W;
-  const long long seg = (long long)b * s.G + g;
-  // CTAs whose range [T c / C, T (c+1) / C) meets [P, P + W)
-  int c0 = 0, c1 = -1;
-  if (W > 0 && T > 0) {
-    c0 = (int)((__int128)P * C / T);
-    while (c0 > 0 && (long long)((__int128)T * c0 / C) > P) --c0;
-    while ((long long)((__int128)T * (c0 + 1) / C) <= P) ++c0;
-    c1 = (int)((__int128)(P + W - 1) * C / T);
-    while (c1 + 1 < C && (long long)((__int128)T * (c1 + 1) / C) <= P + W - 1) ++c1;
-    while (c1 > c0 && (long long)((__int128)T * c1 / C) > P + W - 1) --c1;
-  }
-  const float scale = kLog2e * rsqrtf((float)kHeadDim);
-  pdl_wait();   // the partials come from the preceding decode grid
-  // exact tail scores (n_tail <= 64 on this path)
-  for (int i = warp; i < s.grp * n_tail; i += blockDim.x / 32) {
-    const int h = i / n_tail, t = i % n_tail;
-    const __nv_bfloat16* tk = tail_k + (((long long)b * s.G + g) * n_tail + t) * kHeadDim;
-    float a = 0.f;
-#pragma unroll
-    for (int k = 0; k < 4; ++k) a = fmaf(qrow[h][lane * 4 + k], __bfloat162float(tk[lane * 4 + k]), a);
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) a += __shfl_xor_sync(0xffffffffu, a, o);
-    if (lane == 0) tsc[h][t] = a * scale;
-  }
-  __syncthreads();
-  // per head (one warp each): max over partials and tail, then the softmax denominator
-  for (int h = warp; h < s.grp; h += blockDim.x / 32) {
-    float mx = -INFINITY;
-    for (int cc = c0 + lane; cc <= c1; cc += 32)
-      mx = fmaxf(mx, part[((cc + seg) * kHeadsPad + h) * kPartStride + kHeadDim]);
-    for (int t = lane; t < n_tail; t += 32) mx = fmaxf(mx, tsc[h][t]);
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-    float l = 0.f;
-    for (int cc = c0 + lane; cc <= c1; cc += 32) {
-      const float* pp = part + ((cc + seg) * kHeadsPad + h) * kPartStride;
-      if (pp[kHeadDim] != -INFINITY) l = fmaf(pp[kHeadDim + 1], exp2f(pp[kHeadDim] - mx), l);
-    }
-    __syncwarp();
-    for (int t = lane; t < n_tail; t += 32) {
-      const float w = exp2f(tsc[h][t] - mx);
-      tsc[h][t] = w;
-      l += w;
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
-    if (lane == 0) { hm[h] = mx; hl[h] = l; }
-  }
-  __syncthreads();
-  for (int i = tid; i < s.grp * kHeadDim; i += blockDim.x) {
-    const int h = i / kHeadDim, j = i % kHeadDim;
-    float o = 0.f;
-    for (int cc = c0; cc <= c1; ++cc) {
-      const float* pp = part + ((cc + seg) * kHeadsPad + h) * kPartStride;
-      if (pp[kHeadDim] != -INFINITY) o = fmaf(pp[j], exp2f(pp[kHeadDim] - hm[h]), o);
-    }
-    ot[h][j] = o;
-  }
-  __syncthreads();
-  for (int i = tid; i < s.grp * kHeadDim; i += blockDim.x) {
-    const int h = i / kHeadDim, col = i % kHeadDim;
-    float y = 0.f;
-#pragma unroll 8
-    for (int j = 0; j < kHeadDim; ++j) y = fmaf(__bfloat162float(us[j * kHeadDim + col]), ot[h][j], y);
-    for (int t = 0; t < n_tail; ++t)
-      y = fmaf(tsc[h][t], __bfloat162float(tail_v[(((long long)b * s.G + g) * n_tail + t) * kHeadDim + col]), y);
-    out[((long long)b * s.H + (long long)g * s.grp + h) * kHeadDim + col] = __float2bfloat16_rn(y / hl[h]);
-  }
   pdl_trigger();
 }
 
@@ -602,12 +792,17 @@ decode_combine_mma_kernel(const float* __restrict__ part, const int64_t* __restr
 
 size_t decode_mma_smem_bytes() { return (size_t)NW * ST * STAGE + sizeof(SegSmem); }
 
+// partials, then one completion counter per (sequence, head) segment
 size_t decode_mma_part_bytes(const Shape& s, int num_sms) {
-  return (size_t)(num_sms + (size_t)s.B * s.G) * kHeadsPad * kPartStride * sizeof(float);
+  const size_t p = (size_t)(num_sms + (size_t)s.B * s.G) * kHeadsPad * kPartStride * sizeof(float);
+  return ((p + 255) & ~size_t(255)) + (size_t)s.B * s.G * sizeof(int);
 }
 
-bool decode_mma_supported(const Shape& s, int n_tail) {
-  return s.dtype == VARRATE_BF16 && s.B <= 64 && n_tail <= 64;
+bool decode_mma_supported(const Shape& s, int n_tail, int num_sms) {
+  // the cost line (at most B G cap elements) times the grid size must stay below 2^62
+  const unsigned long long line = (unsigned long long)s.B * s.G * ((unsigned long long)s.cap + kSegCost);
+  return s.dtype == VARRATE_BF16 && s.B <= 64 && n_tail <= 64 && num_sms >= 1 &&
+         num_sms <= kMaxCtas && line <= (1ull << 62) / (unsigned long long)num_sms;
 }
 
 int launch_decode_mma(const Shape& s, const varrate_packed& c, const void* basis_k,
@@ -616,8 +811,8 @@ int launch_decode_mma(const Shape& s, const varrate_packed& c, const void* basis
                       int num_sms, cudaStream_t st) {
   const size_t smem = decode_mma_smem_bytes();
   cudaFuncSetAttribute(decode_mma_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  // both grids may be scheduled while their predecessor drains (programmatic dependent launch);
-  // each waits on griddepcontrol.wait before touching what its predecessor wrote
+  // the grid may be scheduled while its predecessor drains (programmatic dependent launch); it
+  // waits on griddepcontrol.wait before touching anything an earlier operation wrote
   cudaLaunchAttribute pdl[1];
   pdl[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   pdl[0].val.programmaticStreamSerializationAllowed = 1;
@@ -628,17 +823,15 @@ int launch_decode_mma(const Shape& s, const varrate_packed& c, const void* basis
   lc.stream = st;
   lc.attrs = pdl;
   lc.numAttrs = 1;
+  const size_t pbytes = ((size_t)(num_sms + (size_t)s.B * s.G) * kHeadsPad * kPartStride * sizeof(float) + 255) & ~size_t(255);
+  int* seg_done = reinterpret_cast<int*>(reinterpret_cast<char*>(part) + pbytes);
+  cudaMemsetAsync(seg_done, 0, (size_t)s.B * s.G * sizeof(int), st);
   cudaLaunchKernelEx(&lc, decode_mma_kernel, (const __nv_bfloat16*)c.coef, (const int32_t*)c.bucket_count,
                      (const int64_t*)c.bucket_base, (const __nv_bfloat16*)basis_k,
-                     (const __nv_bfloat16*)q, part, dev_status, s, layer);
-  lc.gridDim = dim3(s.G, s.B);
-  lc.blockDim = dim3(256);
-  lc.dynamicSmemBytes = 0;
-  cudaLaunchKernelEx(&lc, decode_combine_mma_kernel, (const float*)part, (const int64_t*)c.bucket_base,
-                     (const __nv_bfloat16*)q, (const __nv_bfloat16*)basis_v,
+                     (const __nv_bfloat16*)basis_v, (const __nv_bfloat16*)q,
                      (const __nv_bfloat16*)tail_k, (const __nv_bfloat16*)tail_v, n_tail,
-                     (__nv_bfloat16*)out, s, layer, num_sms);
-  return 2;
+                     (__nv_bfloat16*)out, part, seg_done, dev_status, s, layer);
+  return 1;
 }
 
 }  // namespace vr

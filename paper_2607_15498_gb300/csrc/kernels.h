@@ -50,7 +50,7 @@ size_t decode_ws_bytes(const Shape& s, int num_sms);
 // bf16 tensor-core decode (decode_mma.cu)
 size_t decode_mma_smem_bytes();
 size_t decode_mma_part_bytes(const Shape& s, int num_sms);
-bool decode_mma_supported(const Shape& s, int n_tail);
+bool decode_mma_supported(const Shape& s, int n_tail, int num_sms);
 int launch_decode_mma(const Shape& s, const varrate_packed& c, const void* basis_k,
                       const void* basis_v, const void* q, int layer, const void* tail_k,
                       const void* tail_v, int n_tail, void* out, int32_t* dev_status, float* part,
