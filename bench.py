@@ -58,17 +58,23 @@ def measured_traffic():
     import hashlib
     import re
     prof = os.path.join(ROOT, "profiles", "decode_mma_llama32.md")
-    src = os.path.join(ROOT, "paper_2607_15498_gb300", "csrc", "decode_mma.cu")
-    if not (os.path.exists(prof) and os.path.exists(src)):
+    if not os.path.exists(prof):
         return None
     text = open(prof).read()
     m_bytes = re.search(r"traffic_bytes_per_launch:\s*([0-9]+)", text)
     m_sha = re.search(r"kernel_source_sha256:\s*([0-9a-f]{64})", text)
-    if not (m_bytes and m_sha):
-        return None
-    if hashlib.sha256(open(src, "rb").read()).hexdigest() != m_sha.group(1):
+    if not (m_bytes and m_sha) or kernel_source_sha256() != m_sha.group(1):
         return None
     return int(m_bytes.group(1))
+
+
+def kernel_source_sha256():
+    """sha256 over the decode kernel's sources (decode_mma.cu, then common.cuh)."""
+    import hashlib
+    h = hashlib.sha256()
+    for name in ("decode_mma.cu", "common.cuh"):
+        h.update(open(os.path.join(ROOT, "paper_2607_15498_gb300", "csrc", name), "rb").read())
+    return h.hexdigest()
 
 
 def dist_env():
@@ -425,7 +431,7 @@ def main():
                 decode_ms_per_step=round(1e3 * dec_s / K / args.decode_steps, 4),
                 decode_frac_of_hbm_peak=round(dec_gbs / world / peak, 4),
                 decode_frac_of_nominal_8tbs=round(dec_gbs / world / 8000.0, 4),
-                roofline={"bound": "hbm", "kernel": "varrate_decode_attn (rotate + split + combine)",
+                roofline={"bound": "hbm", "kernel": "decode_mma_kernel (one fused launch per layer call)",
                           "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
                           "frac": round(achieved / peak, 4), "traffic": measured_traffic(),
                           "peak_source": f"{peak_kind} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)"
