@@ -4,7 +4,7 @@
 //
 // One CTA owns a range of bucketed slots of one (sequence, layer, head, K-or-V) stream and runs
 // three warp roles over a 5-stage ring of 128-slot tiles:
-//   producers (2 warps)  for tile i: token t = perm[slot]; rank r and in-bucket position p follow
+//   producers (4 warps)  for tile i: token t = perm[slot]; rank r and in-bucket position p follow
 //                        from the slot alone (tokens sit in slot order inside a bucket: r is found
 //                        by a prefix search over the bucket counts, p = slot - bucket start). Token
 //                        rows (256 B) are gathered with 16-byte cp.async, 16 lanes per row, into a
@@ -31,8 +31,11 @@ constexpr int NST = 5;                     // operand stages
 constexpr int NMETA = NST + 2;             // metadata ring (outlives the epilogue of its tile)
 constexpr int LAG = 2;                     // copy groups kept in flight behind the signalled one
 constexpr int TILE_BYTES = TM * kHeadDim * 2;
-constexpr int kEpi = 4, kProd = 2;         // warps
+constexpr int kEpi = 4, kProd = 4;         // warps
 constexpr int kThreads = (kEpi + kProd + 1) * 32;
+constexpr int kProdThreads = kProd * 32;
+constexpr int kRowsPer = TM / kProdThreads;     // metadata rows per producer thread
+static_assert(TM % kProdThreads == 0 && kProdThreads % 16 == 0, "producer split");
 constexpr uint32_t kWaitTries = 1u << 22;  // bounded mbarrier polls
 
 struct ProjSmem {
@@ -109,7 +112,7 @@ project_tc_kernel(const __nv_bfloat16* __restrict__ k, const __nv_bfloat16* __re
 
   if (warp >= kEpi && warp < kEpi + kProd) {
     // ------------------------------------------------------------------ producers
-    const int pt = tid - kEpi * 32;            // 0 .. 63
+    const int pt = tid - kEpi * 32;            // 0 .. kProdThreads - 1
     bool bad = false;
     auto signal = [&](int j) {                 // this thread's copies of tile j have landed
       fence_proxy_async_smem();
@@ -120,12 +123,17 @@ project_tc_kernel(const __nv_bfloat16* __restrict__ k, const __nv_bfloat16* __re
       const int64_t slot = s_begin + (int64_t)i * TM + row;
       return (i < n_tiles && slot < s_end) ? perm[bl * s.N + slot] : -1;
     };
-    int t_next[2] = {perm_of(0, pt), perm_of(0, pt + 64)};
+    int t_next[kRowsPer];
+#pragma unroll
+    for (int h = 0; h < kRowsPer; ++h) t_next[h] = perm_of(0, pt + kProdThreads * h);
     for (int i = 0; i < n_tiles; ++i) {
       const int st = i % NST, mt = i % NMETA;
-      const int t_cur[2] = {t_next[0], t_next[1]};
-      t_next[0] = perm_of(i + 1, pt);
-      t_next[1] = perm_of(i + 1, pt + 64);
+      int t_cur[kRowsPer];
+#pragma unroll
+      for (int h = 0; h < kRowsPer; ++h) {
+        t_cur[h] = t_next[h];
+        t_next[h] = perm_of(i + 1, pt + kProdThreads * h);
+      }
       if (!bad && !mbar_wait_bounded(&sm.empty[st], ((i / NST) & 1) ^ 1, kWaitTries)) { sm.err = 1; bad = true; }
       // bucket of the tile's first slot (same search in every lane: broadcast reads), then a short
       // forward scan per row: buckets are in slot order
@@ -140,8 +148,8 @@ project_tc_kernel(const __nv_bfloat16* __restrict__ k, const __nv_bfloat16* __re
         r0 = lo;
       }
 #pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        const int row = pt + 64 * h;
+      for (int h = 0; h < kRowsPer; ++h) {
+        const int row = pt + kProdThreads * h;
         const int slot = slot0 + row;
         const int t = t_cur[h];
         int r = 0, p = 0;
@@ -158,8 +166,8 @@ project_tc_kernel(const __nv_bfloat16* __restrict__ k, const __nv_bfloat16* __re
       const uint32_t dst = stage0 + st * TILE_BYTES;
       const int c = pt & 15;
 #pragma unroll
-      for (int q = 0; q < TM / 4; ++q) {
-        const int row = (pt >> 4) + 4 * q;
+      for (int q = 0; q < TM * 16 / kProdThreads; ++q) {
+        const int row = (pt >> 4) + (kProdThreads / 16) * q;
         const int t = sm.tok[mt][row];
         const __nv_bfloat16* src = x + (int64_t)(t < 0 ? 0 : t) * kHeadDim + c * 8;
         cp_async16(dst + sw128_offset(row, c, TM), src, t >= 0 ? 16u : 0u);
