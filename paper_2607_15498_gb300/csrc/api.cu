@@ -159,7 +159,8 @@ varrate_status varrate_pack(const varrate_config* cfg, const void* k, const void
   if (st != VARRATE_OK) return st;
   if (!k || !v || !basis_k || !basis_v || !packed_ok(cfg, out)) return VARRATE_ERR_ARG;
   const Shape s = make_shape(cfg, out->cap_elems);
-  vr::launch_pack(s, k, v, basis_k, basis_v, *out, dev_status, num_sms(), (cudaStream_t)stream);
+  if (vr::launch_pack(s, k, v, basis_k, basis_v, *out, dev_status, num_sms(), (cudaStream_t)stream) < 0)
+    return VARRATE_ERR_CUDA;
   return launched();
 }
 
@@ -185,7 +186,7 @@ varrate_status varrate_encode(const varrate_config* cfg, const void* q_win, cons
   if (cfg->mode == VARRATE_SALIENCE && vr::launch_salience(s, q_win, k, sal, w, dev_status, sms, cs) < 0)
     return VARRATE_ERR_CUDA;
   vr::launch_allocate(s, sal, out->ranks, realized, dev_status, cs);
-  vr::launch_pack(s, k, v, basis_k, basis_v, *out, dev_status, sms, cs);
+  if (vr::launch_pack(s, k, v, basis_k, basis_v, *out, dev_status, sms, cs) < 0) return VARRATE_ERR_CUDA;
   return launched();
 }
 

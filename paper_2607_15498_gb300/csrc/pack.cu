@@ -227,7 +227,8 @@ int launch_pack(const Shape& s, const void* k, const void* v, const void* basis_
     using T = __nv_bfloat16;
     pack_tables_kernel<T><<<s.B * s.L, 1024, 0, st>>>(out.ranks, out.bucket_count, out.bucket_base,
                                                       out.perm, out.pos, (T*)out.coef, dev_status, s);
-    return 1 + launch_project_tc(s, k, v, basis_k, basis_v, out, dev_status, num_sms, st);
+    const int np = launch_project_tc(s, k, v, basis_k, basis_v, out, dev_status, num_sms, st);
+    return np < 0 ? -1 : 1 + np;
   } else {
     using T = float;
     pack_tables_kernel<T><<<s.B * s.L, 1024, 0, st>>>(out.ranks, out.bucket_count, out.bucket_base,

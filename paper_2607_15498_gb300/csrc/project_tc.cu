@@ -2,22 +2,22 @@
 // (Algorithm 1's projection c_t = U x_t, Eq. 5 with the anchor mean at 0), written straight into
 // the rank-bucketed layout.
 //
-// One CTA owns a range of bucketed slots of one (sequence, layer, head, K-or-V) stream and runs
-// three warp roles over a 5-stage ring of 128-slot tiles:
-//   producers (4 warps)  for tile i: token t = perm[slot]; rank r and in-bucket position p follow
-//                        from the slot alone (tokens sit in slot order inside a bucket: r is found
-//                        by a prefix search over the bucket counts, p = slot - bucket start). Token
-//                        rows (256 B) are gathered with 16-byte cp.async, 16 lanes per row, into a
-//                        128 x 128 bf16 tile in the K-major 128-byte-swizzled layout the tensor core
-//                        reads; once a tile's copies have landed the producers fence the async proxy
-//                        and arrive on the stage's mbarrier (two tiles stay in flight behind it).
-//   mma (1 thread)       8 x tcgen05.mma (M = 128 slots, N = 128 coefficients, K = 16) with U
-//                        (128 x 128, resident in shared memory) as B, into one of two TMEM
-//                        accumulators; tcgen05.commit frees the stage and hands the accumulator on.
-//   epilogue (4 warps)   warp w reads TMEM lanes 32w..32w+31 (row = slot) 32 columns at a time and
-//                        stores coefficient j < r of the slot's token in the tiled bucket layout
-//                        (coef_offset): lanes of one 8-slot group write consecutive addresses.
+// One CTA owns a range of tokens (in sequence order) of one (sequence, layer, head, K-or-V) stream
+// and runs three warp roles over a 5-stage ring of 128-token tiles:
+//   producer (1 thread)  two TMA tile loads per tile (64 columns x 128 rows each, 128-byte swizzle:
+//                        the K-major operand layout of the tensor core) of 128 consecutive token
+//                        rows; the K / V tensors are read once, front to back;
+//   mma (1 thread)       8 x tcgen05.mma (M = 128 tokens, N = 128 coefficients, K = 16) with U
+//                        (128 x 128, resident in shared memory) as B, into one of four TMEM
+//                        accumulators; tcgen05.commit frees the stage and hands the accumulator on;
+//   epilogue (16 warps)  four groups of four take the tiles round-robin (each group covers the 128 TMEM
+//                        lanes); thread = token: reads its rank r and in-bucket position p (coalesced),
+//                        then its TMEM row 32 columns at a time, and stores coefficient j < r at
+//                        its slot of bucket r (coef_offset). Consecutive tokens of one rank hold
+//                        consecutive slots, so each store instruction writes a few 16-byte runs.
 // Every mbarrier wait is bounded; a timeout raises VARRATE_ERR_TIMEOUT.
+#include <cudaTypedefs.h>
+
 #include "common.cuh"
 #include "kernels.h"
 
@@ -26,36 +26,30 @@ namespace vr {
 namespace {
 
 constexpr int kMaxR = kHeadDim;
-constexpr int TM = 128;                    // slots per tile
+constexpr int TM = 128;                    // tokens per tile
 constexpr int NST = 5;                     // operand stages
-constexpr int NMETA = NST + 2;             // metadata ring (outlives the epilogue of its tile)
-constexpr int LAG = 2;                     // copy groups kept in flight behind the signalled one
 constexpr int TILE_BYTES = TM * kHeadDim * 2;
-constexpr int kEpi = 4, kProd = 4;         // warps
-constexpr int kThreads = (kEpi + kProd + 1) * 32;
-constexpr int kProdThreads = kProd * 32;
-constexpr int kRowsPer = TM / kProdThreads;     // metadata rows per producer thread
-static_assert(TM % kProdThreads == 0 && kProdThreads % 16 == 0, "producer split");
+constexpr int NGRP = 4;                    // epilogue groups of four warps (tiles round-robin)
+constexpr int kEpi = 4 * NGRP;             // epilogue warps
+constexpr int NACC = 4;                    // TMEM accumulators of 128 columns (all 512 columns)
+constexpr int kThreads = (kEpi + 2) * 32;  // + producer warp + MMA warp
 constexpr uint32_t kWaitTries = 1u << 22;  // bounded mbarrier polls
 
 struct ProjSmem {
-  uint64_t full[NST], empty[NST], tfull[2], tempty[2];
+  uint64_t full[NST], empty[NST], tfull[NACC], tempty[NACC];
   uint32_t tmem_base;
   int err;
-  int tok[NMETA][TM];
-  int rk[NMETA][TM];
-  int ps[NMETA][TM];
   int n8[kMaxR + 1];
-  int slot_start[kMaxR + 2];   // first bucketed slot of rank r (exclusive prefix of the counts)
   long long base[kMaxR + 2];
 };
 
 __global__ void __launch_bounds__(kThreads, 1)
-project_tc_kernel(const __nv_bfloat16* __restrict__ k, const __nv_bfloat16* __restrict__ v,
+project_tc_kernel(const __grid_constant__ CUtensorMap tk, const __grid_constant__ CUtensorMap tv,
                   const __nv_bfloat16* __restrict__ basis_k, const __nv_bfloat16* __restrict__ basis_v,
                   const int32_t* __restrict__ bucket_count, const int64_t* __restrict__ bucket_base,
-                  const int32_t* __restrict__ perm, __nv_bfloat16* __restrict__ coef,
-                  int32_t* __restrict__ dev_status, Shape s, int64_t chunk) {
+                  const uint8_t* __restrict__ ranks, const int32_t* __restrict__ pos,
+                  __nv_bfloat16* __restrict__ coef, int32_t* __restrict__ dev_status, Shape s,
+                  int64_t chunk) {
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   // 1024-byte alignment for the swizzled operand tiles
   unsigned char* smem = smem_raw + ((1024 - (smem_addr(smem_raw) & 1023)) & 1023);
@@ -72,15 +66,7 @@ project_tc_kernel(const __nv_bfloat16* __restrict__ k, const __nv_bfloat16* __re
     if (r <= kMaxR) sm.n8[r] = (int)pad8(bucket_count[bl * (kMaxR + 1) + r]);
     sm.base[r] = bucket_base[bl * (kMaxR + 2) + r];
   }
-  if (tid == 0) {
-    sm.err = 0;
-    int acc = 0;
-    for (int r = 0; r <= kMaxR; ++r) {
-      sm.slot_start[r] = acc;
-      acc += bucket_count[bl * (kMaxR + 1) + r];
-    }
-    sm.slot_start[kMaxR + 1] = acc;
-  }
+  if (tid == 0) sm.err = 0;
   __syncthreads();
   if (sm.base[kMaxR + 1] > s.cap || sm.base[kMaxR + 1] < 0) return;   // reported by pack_tables
 
@@ -91,103 +77,48 @@ project_tc_kernel(const __nv_bfloat16* __restrict__ k, const __nv_bfloat16* __re
     *reinterpret_cast<uint4*>(u_tile + sw128_offset(row, c, TM)) =
         __ldg(reinterpret_cast<const uint4*>(U + (int64_t)row * kHeadDim) + c);
   }
-  if (warp == kEpi + kProd && lane == 0) {
-    for (int i = 0; i < NST; ++i) { mbar_init(&sm.full[i], kProd * 32); mbar_init(&sm.empty[i], 1); }
-    for (int i = 0; i < 2; ++i) { mbar_init(&sm.tfull[i], 1); mbar_init(&sm.tempty[i], kEpi); }
+  if (warp == kEpi && lane == 0) {
+    for (int i = 0; i < NST; ++i) { mbar_init(&sm.full[i], 1); mbar_init(&sm.empty[i], 1); }
+    for (int i = 0; i < NACC; ++i) { mbar_init(&sm.tfull[i], 1); mbar_init(&sm.tempty[i], 4); }
     fence_mbar_init();
   }
-  if (warp == 0) tmem_alloc(&sm.tmem_base, 256);
+  if (warp == 0) tmem_alloc(&sm.tmem_base, NACC * kHeadDim);
   fence_proxy_async_smem();
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = sm.tmem_base;
 
-  const __nv_bfloat16* x = (kv ? v : k) + (bl * s.G + g) * s.N * kHeadDim;
   __nv_bfloat16* out = coef + ((bl * s.G + g) * 2 + kv) * s.cap;
-  const int64_t s_begin = blockIdx.x * chunk;
-  const int64_t s_end = min(s.N, s_begin + chunk);
-  const int n_tiles = (int)((s_end - s_begin + TM - 1) / TM);
+  const int64_t t_begin = blockIdx.x * chunk;
+  const int64_t t_end = min(s.N, t_begin + chunk);
+  const int n_tiles = (int)((t_end - t_begin + TM - 1) / TM);
   const uint32_t stage0 = smem_addr(stages), u_addr = smem_addr(u_tile);
 
-  if (warp >= kEpi && warp < kEpi + kProd) {
-    // ------------------------------------------------------------------ producers
-    const int pt = tid - kEpi * 32;            // 0 .. kProdThreads - 1
-    bool bad = false;
-    auto signal = [&](int j) {                 // this thread's copies of tile j have landed
-      fence_proxy_async_smem();
-      mbar_arrive(&sm.full[j % NST]);
-    };
-    // perm of this thread's two rows, one tile ahead of its use
-    auto perm_of = [&](int i, int row) -> int {
-      const int64_t slot = s_begin + (int64_t)i * TM + row;
-      return (i < n_tiles && slot < s_end) ? perm[bl * s.N + slot] : -1;
-    };
-    int t_next[kRowsPer];
-#pragma unroll
-    for (int h = 0; h < kRowsPer; ++h) t_next[h] = perm_of(0, pt + kProdThreads * h);
-    for (int i = 0; i < n_tiles; ++i) {
-      const int st = i % NST, mt = i % NMETA;
-      int t_cur[kRowsPer];
-#pragma unroll
-      for (int h = 0; h < kRowsPer; ++h) {
-        t_cur[h] = t_next[h];
-        t_next[h] = perm_of(i + 1, pt + kProdThreads * h);
-      }
-      if (!bad && !mbar_wait_bounded(&sm.empty[st], ((i / NST) & 1) ^ 1, kWaitTries)) { sm.err = 1; bad = true; }
-      // bucket of the tile's first slot (same search in every lane: broadcast reads), then a short
-      // forward scan per row: buckets are in slot order
-      const int slot0 = (int)(s_begin + (int64_t)i * TM);
-      int r0 = 0;
-      {
-        int lo = 0, hi = kMaxR + 1;            // slot_start[lo] <= slot0 < slot_start[hi]
-        while (hi - lo > 1) {
-          const int mid = (lo + hi) >> 1;
-          if (sm.slot_start[mid] <= slot0) lo = mid; else hi = mid;
-        }
-        r0 = lo;
-      }
-#pragma unroll
-      for (int h = 0; h < kRowsPer; ++h) {
-        const int row = pt + kProdThreads * h;
-        const int slot = slot0 + row;
-        const int t = t_cur[h];
-        int r = 0, p = 0;
-        if (t >= 0) {
-          r = r0;
-          while (sm.slot_start[r + 1] <= slot) ++r;
-          p = slot - sm.slot_start[r];
-        }
-        sm.tok[mt][row] = t;
-        sm.rk[mt][row] = r;
-        sm.ps[mt][row] = p;
-      }
-      named_sync(1, kProd * 32);               // metadata of every row of the tile is visible
-      const uint32_t dst = stage0 + st * TILE_BYTES;
-      const int c = pt & 15;
-#pragma unroll
-      for (int q = 0; q < TM * 16 / kProdThreads; ++q) {
-        const int row = (pt >> 4) + (kProdThreads / 16) * q;
-        const int t = sm.tok[mt][row];
-        const __nv_bfloat16* src = x + (int64_t)(t < 0 ? 0 : t) * kHeadDim + c * 8;
-        cp_async16(dst + sw128_offset(row, c, TM), src, t >= 0 ? 16u : 0u);
-      }
-      cp_async_commit();
-      if (i >= LAG) {
-        cp_async_wait<LAG>();
-        signal(i - LAG);
+  if (warp == kEpi) {
+    // ------------------------------------------------------------------ producer
+    if (lane == 0) {
+      const CUtensorMap* map = kv ? &tv : &tk;
+      const int row0 = (int)((bl * s.G + g) * s.N + t_begin);   // rows of the [B L G N][128] view
+      for (int i = 0; i < n_tiles; ++i) {
+        const int st = i % NST;
+        if (!mbar_wait_bounded(&sm.empty[st], ((i / NST) & 1) ^ 1, kWaitTries)) { sm.err = 1; break; }
+        const uint32_t dst = stage0 + st * TILE_BYTES;
+        mbar_arrive_expect_tx(&sm.full[st], TILE_BYTES);
+        // rows past the stream's end belong to the next stream (or read as zero): their results
+        // are never stored
+        tma_load_2d(dst, map, 0, row0 + i * TM, &sm.full[st]);
+        tma_load_2d(dst + TM * 128, map, 64, row0 + i * TM, &sm.full[st]);
       }
     }
-    cp_async_wait<0>();
-    for (int j = max(0, n_tiles - LAG); j < n_tiles; ++j) signal(j);
-  } else if (warp == kEpi + kProd) {
+  } else if (warp == kEpi + 1) {
     // ------------------------------------------------------------------ MMA issuer
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_bf16_f32(TM, kHeadDim);
       for (int i = 0; i < n_tiles; ++i) {
-        const int st = i % NST, b = i & 1;
+        const int st = i % NST, b = i % NACC;
         if (!mbar_wait_bounded(&sm.full[st], (i / NST) & 1, kWaitTries) ||
-            !mbar_wait_bounded(&sm.tempty[b], ((i >> 1) & 1) ^ 1, kWaitTries)) { sm.err = 1; break; }
+            !mbar_wait_bounded(&sm.tempty[b], ((i / NACC) & 1) ^ 1, kWaitTries)) { sm.err = 1; break; }
         tc_fence_after();
         const uint32_t a0 = stage0 + st * TILE_BYTES;
         const uint32_t d = tmem + (uint32_t)(b * kHeadDim);
@@ -203,20 +134,33 @@ project_tc_kernel(const __nv_bfloat16* __restrict__ k, const __nv_bfloat16* __re
   } else {
     // ------------------------------------------------------------------ epilogue
     bool bad = false;
-    for (int i = 0; i < n_tiles; ++i) {
-      const int b = i & 1, mt = i % NMETA;
-      if (!bad && !mbar_wait_bounded(&sm.tfull[b], (i >> 1) & 1, kWaitTries)) { sm.err = 1; bad = true; }
+    const int eg = warp >> 2, row = tid & (TM - 1);   // epilogue group (tiles eg, eg + NGRP, ...), token row
+    // rank and bucket position of this thread's token, one tile of its group ahead of its use
+    auto meta = [&](int i, int& r, int& p) {
+      const int64_t t = t_begin + (int64_t)i * TM + row;
+      const bool ok = i < n_tiles && t < t_end;
+      r = ok ? (int)ranks[bl * s.N + t] : 0;
+      p = ok ? pos[bl * s.N + t] : 0;
+    };
+    int r_next, p_next;
+    meta(eg, r_next, p_next);
+    for (int i = eg; i < n_tiles; i += NGRP) {
+      const int b = i % NACC;
+      const int r = r_next, p = p_next;
+      meta(i + NGRP, r_next, p_next);
+      const bool valid = r >= s.r_min && r <= s.r_max;   // a token of this stream, rank in range
+      if (!bad && !mbar_wait_bounded(&sm.tfull[b], (i / NACC) & 1, kWaitTries)) { sm.err = 1; bad = true; }
       tc_fence_after();
-      const int t = sm.tok[mt][tid], r = sm.rk[mt][tid], p = sm.ps[mt][tid];
-      const int rmax_w = __reduce_max_sync(0xffffffffu, t >= 0 ? r : 0);
+      const int rmax_w = __reduce_max_sync(0xffffffffu, valid ? r : 0);
       // this slot's position in its 128-slot tile (coef_offset): the row of coefficient j starts at
       // tile + j * tl, the slot's 8-group rotates by one position per row
+      const int rr = valid ? r : s.r_min;
       const long long p0 = ((long long)p >> 7) << 7;
-      const int tl = (int)min(128LL, (long long)sm.n8[r] - p0);
+      const int tl = (int)min(128LL, (long long)sm.n8[rr] - p0);
       const int ng = max(tl >> 3, 1);
       const int pl = p - (int)p0;
-      __nv_bfloat16* tile = out + sm.base[r] + p0 * r + (pl & 7);
-      const uint32_t taddr = tmem + (uint32_t)(b * kHeadDim) + ((uint32_t)(warp * 32) << 16);
+      __nv_bfloat16* tile = out + sm.base[rr] + p0 * rr + (pl & 7);
+      const uint32_t taddr = tmem + (uint32_t)(b * kHeadDim) + ((uint32_t)((warp & 3) * 32) << 16);
       int grp = (pl >> 3) % ng;
 #pragma unroll
       for (int cb = 0; cb < kHeadDim / 32; ++cb) {
@@ -226,7 +170,7 @@ project_tc_kernel(const __nv_bfloat16* __restrict__ k, const __nv_bfloat16* __re
 #pragma unroll
         for (int jj = 0; jj < 32; ++jj) {
           const int j = cb * 32 + jj;
-          if (!bad && t >= 0 && j < r) tile[(long long)j * tl + grp * 8] = __float2bfloat16_rn(vals[jj]);
+          if (!bad && valid && j < r) tile[(long long)j * tl + grp * 8] = __float2bfloat16_rn(vals[jj]);
           grp = (grp + 1 == ng) ? 0 : grp + 1;
         }
       }
@@ -237,7 +181,7 @@ project_tc_kernel(const __nv_bfloat16* __restrict__ k, const __nv_bfloat16* __re
   }
   tc_fence_before();
   __syncthreads();
-  if (warp == 0) tmem_dealloc(tmem, 256);
+  if (warp == 0) tmem_dealloc(tmem, NACC * kHeadDim);
   if (tid == 0 && sm.err) raise_status(dev_status, VARRATE_ERR_TIMEOUT);
 }
 
@@ -245,9 +189,15 @@ project_tc_kernel(const __nv_bfloat16* __restrict__ k, const __nv_bfloat16* __re
 
 size_t project_tc_smem_bytes() { return 1024 + (size_t)(1 + NST) * TILE_BYTES + sizeof(ProjSmem); }
 
+bool make_tmap_rows_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint32_t box_rows);
+
 int launch_project_tc(const Shape& s, const void* k, const void* v, const void* basis_k,
                       const void* basis_v, const varrate_packed& out, int32_t* dev_status,
                       int num_sms, cudaStream_t st) {
+  const uint64_t rows = (uint64_t)s.B * s.L * s.G * s.N;
+  if (rows > (uint64_t)INT32_MAX) return -1;   // TMA row coordinates are 32-bit
+  CUtensorMap tk, tv;
+  if (!make_tmap_rows_bf16(&tk, k, rows, TM) || !make_tmap_rows_bf16(&tv, v, rows, TM)) return -1;
   const int64_t units = (int64_t)s.B * s.L * s.G * 2;
   int64_t n = (2LL * num_sms + units - 1) / units;
   int64_t chunk = (s.N + n - 1) / n;
@@ -256,9 +206,8 @@ int launch_project_tc(const Shape& s, const void* k, const void* v, const void* 
   const size_t smem = project_tc_smem_bytes();
   cudaFuncSetAttribute(project_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   project_tc_kernel<<<dim3(n_chunks, s.G * 2, s.B * s.L), kThreads, smem, st>>>(
-      (const __nv_bfloat16*)k, (const __nv_bfloat16*)v, (const __nv_bfloat16*)basis_k,
-      (const __nv_bfloat16*)basis_v, out.bucket_count, out.bucket_base, out.perm,
-      (__nv_bfloat16*)out.coef, dev_status, s, chunk);
+      tk, tv, (const __nv_bfloat16*)basis_k, (const __nv_bfloat16*)basis_v, out.bucket_count,
+      out.bucket_base, out.ranks, out.pos, (__nv_bfloat16*)out.coef, dev_status, s, chunk);
   return 1;
 }
 
