@@ -25,7 +25,8 @@
  *    both cases.
  *  - Limits: head_dim == 128, 1 <= group <= 8, 1 <= window and group * window <= 256,
  *    window <= n_ctx < 2^31, 1 <= r_min <= head_dim, pool_len odd in [1, 31],
- *    0 < budget_frac <= 1.
+ *    0 < budget_frac <= 1; in bf16, batch * n_layers * n_kv_heads * n_ctx < 2^31 (the K and V
+ *    tensors are read through TMA tensor maps with 32-bit row coordinates).
  *
  * Notation: B = batch (sequences), L = n_layers, G = n_kv_heads, H = G * group query heads,
  * d = head_dim, N = n_ctx, w = window. The exact set is the last w tokens [N - w, N) (kept at

@@ -26,6 +26,9 @@ varrate_status check(const varrate_config* c) {
   if (c->head_dim != vr::kHeadDim) return VARRATE_ERR_UNSUPPORTED;
   if (c->r_min > c->head_dim) return VARRATE_ERR_ARG;
   if (c->group > 8 || (int64_t)c->group * c->window > 256) return VARRATE_ERR_UNSUPPORTED;
+  if (c->dtype == VARRATE_BF16 &&
+      (int64_t)c->batch * c->n_layers * c->n_kv_heads * c->n_ctx > (int64_t)INT32_MAX)
+    return VARRATE_ERR_UNSUPPORTED;
   return VARRATE_OK;
 }
 
@@ -159,6 +162,7 @@ varrate_status varrate_pack(const varrate_config* cfg, const void* k, const void
   if (st != VARRATE_OK) return st;
   if (!k || !v || !basis_k || !basis_v || !packed_ok(cfg, out)) return VARRATE_ERR_ARG;
   const Shape s = make_shape(cfg, out->cap_elems);
+  if (!vr::pack_ready(s, k, v)) return VARRATE_ERR_CUDA;   // before anything is enqueued
   if (vr::launch_pack(s, k, v, basis_k, basis_v, *out, dev_status, num_sms(), (cudaStream_t)stream) < 0)
     return VARRATE_ERR_CUDA;
   return launched();
@@ -175,6 +179,7 @@ varrate_status varrate_encode(const varrate_config* cfg, const void* q_win, cons
   const size_t need = ws_bytes(cfg, VARRATE_CALL_ENCODE);
   if (ws_bytes_ < need || ws == nullptr) return VARRATE_ERR_WORKSPACE;
   const Shape s = make_shape(cfg, out->cap_elems);
+  if (!vr::pack_ready(s, k, v)) return VARRATE_ERR_CUDA;   // before anything is enqueued
   const int sms = num_sms();
   cudaStream_t cs = (cudaStream_t)stream;
   char* w = static_cast<char*>(ws);

@@ -34,6 +34,9 @@ int launch_allocate(const Shape& s, const float* sal, uint8_t* ranks, int64_t* r
                     int32_t* dev_status, cudaStream_t st);
 
 // ---- step 3: tables + projection
+// Host-side checks of what launch_pack builds before its first launch (bf16: the TMA tensor maps
+// of k and v); false means launch_pack would fail.
+bool pack_ready(const Shape& s, const void* k, const void* v);
 int launch_pack(const Shape& s, const void* k, const void* v, const void* basis_k,
                 const void* basis_v, const varrate_packed& out, int32_t* dev_status,
                 int num_sms, cudaStream_t st);

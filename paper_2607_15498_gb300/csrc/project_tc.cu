@@ -191,6 +191,14 @@ size_t project_tc_smem_bytes() { return 1024 + (size_t)(1 + NST) * TILE_BYTES + 
 
 bool make_tmap_rows_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint32_t box_rows);
 
+bool pack_ready(const Shape& s, const void* k, const void* v) {
+  if (s.dtype != VARRATE_BF16) return true;
+  const uint64_t rows = (uint64_t)s.B * s.L * s.G * s.N;
+  CUtensorMap tk, tv;
+  return rows <= (uint64_t)INT32_MAX && make_tmap_rows_bf16(&tk, k, rows, TM) &&
+         make_tmap_rows_bf16(&tv, v, rows, TM);
+}
+
 int launch_project_tc(const Shape& s, const void* k, const void* v, const void* basis_k,
                       const void* basis_v, const varrate_packed& out, int32_t* dev_status,
                       int num_sms, cudaStream_t st) {
