@@ -4,7 +4,8 @@
 // score every key: S = Q_g K_g^T / sqrt(d), causal inside the window. Two passes over the keys,
 // both fed by TMA (128-byte swizzle) and accumulated in TMEM by tcgen05.mma:
 //   pass 1  (rows x tokens, M = 128 rows, N = 256 tokens): each epilogue thread owns one row and
-//           keeps its running max and sum of 2^(S * log2e / sqrt(d) - max) over its token chunk;
+//           keeps its running max and sum of 2^(S * log2e / sqrt(d) - max) over the tiles of its
+//           epilogue group (two groups take alternate tiles; their partials merge at the end);
 //   pass 2  (tokens x rows, M = 128 tokens, N = M rows rounded up to 32): each epilogue thread owns
 //           one token and sums 2^(S * log2e / sqrt(d) - lse_row) over the rows of one head; the
 //           pool kernel adds the heads in a fixed order (deterministic) and applies the 5-tap mean.
@@ -23,18 +24,19 @@ namespace {
 constexpr uint32_t kTries = 1u << 22;
 
 // ------------------------------------------------------------------------------- pass 1
-constexpr int P1_EPI = 8;               // epilogue warps (2 per TMEM lane quarter)
+constexpr int P1_NGRP = 2;              // epilogue groups of four warps (alternate tiles)
+constexpr int P1_EPI = 4 * P1_NGRP;
 constexpr int P1_THREADS = (P1_EPI + 2) * 32;
 constexpr int P1_TN = 256;              // tokens per tile (MMA N)
-constexpr int P1_ST = 2;                // key stages
+constexpr int P1_ST = 3;                // key stages (2 in flight behind the one in use)
+constexpr int P1_NACC = 512 / P1_TN;    // TMEM accumulators of P1_TN columns
 constexpr int P1_Q = 128 * 256;         // 128 rows x 128 bf16
-constexpr int P1_K = P1_TN * 256;       // 256 tokens x 128 bf16
+constexpr int P1_K = P1_TN * 256;       // 128 tokens x 128 bf16
 
 struct P1Smem {
-  uint64_t full[P1_ST], empty[P1_ST], tfull[2], tempty[2];
+  uint64_t full[P1_ST], empty[P1_ST], tfull[P1_NACC], tempty[P1_NACC];
   uint32_t tmem;
   int err;
-  float m[2][128], l[2][128];
 };
 
 __global__ void __launch_bounds__(P1_THREADS, 1)
@@ -69,7 +71,7 @@ salience_stats_tc_kernel(const __grid_constant__ CUtensorMap tk, const __nv_bflo
   }
   if (warp == P1_EPI + 1 && lane == 0) {
     for (int i = 0; i < P1_ST; ++i) { mbar_init(&sm.full[i], 1); mbar_init(&sm.empty[i], 1); }
-    for (int i = 0; i < 2; ++i) { mbar_init(&sm.tfull[i], 1); mbar_init(&sm.tempty[i], P1_EPI); }
+    for (int i = 0; i < P1_NACC; ++i) { mbar_init(&sm.tfull[i], 1); mbar_init(&sm.tempty[i], 4); }
     sm.err = 0;
     fence_mbar_init();
   }
@@ -80,6 +82,7 @@ salience_stats_tc_kernel(const __grid_constant__ CUtensorMap tk, const __nv_bflo
   tc_fence_after();
   const uint32_t tmem = sm.tmem;
   const int64_t row0 = (bl * s.G + g) * s.N + t_begin;
+  float rm = -INFINITY, rl = 0.f;   // epilogue: running max and sum of this thread's row
 
   if (warp == P1_EPI) {
     if (lane == 0) {                                  // TMA producer
@@ -97,86 +100,89 @@ salience_stats_tc_kernel(const __grid_constant__ CUtensorMap tk, const __nv_bflo
       constexpr uint32_t idesc = idesc_bf16_f32(128, P1_TN);
       const uint32_t qa = smem_addr(qt);
       for (int i = 0; i < n_tiles; ++i) {
-        const int st = i % P1_ST, b = i & 1;
+        const int st = i % P1_ST, b = i % P1_NACC;
         if (!mbar_wait_bounded(&sm.full[st], (i / P1_ST) & 1, kTries) ||
-            !mbar_wait_bounded(&sm.tempty[b], ((i >> 1) & 1) ^ 1, kTries)) { sm.err = 1; break; }
+            !mbar_wait_bounded(&sm.tempty[b], ((i / P1_NACC) & 1) ^ 1, kTries)) { sm.err = 1; break; }
         tc_fence_after();
         const uint32_t kb = smem_addr(kst + st * P1_K);
 #pragma unroll
         for (int ks = 0; ks < kHeadDim / 16; ++ks) {
           const uint32_t ka = (ks >> 2) * 16384 + (ks & 3) * 32;     // Q panel: 128 rows x 128 B
-          const uint32_t kk = (ks >> 2) * (P1_K / 2) + (ks & 3) * 32; // K panel: 256 rows x 128 B
+          const uint32_t kk = (ks >> 2) * (P1_K / 2) + (ks & 3) * 32; // K panel: 128 rows x 128 B
           tc_mma_bf16(tmem + b * P1_TN, sdesc_sw128(qa + ka), sdesc_sw128(kb + kk), idesc, ks > 0);
         }
         tc_commit(&sm.empty[st]);
         tc_commit(&sm.tfull[b]);
       }
     }
-  } else {                                            // epilogue: one row, half of the columns
-    const int quarter = warp & 3, half = warp >> 2;
+  } else {                                            // epilogue: one row, alternate tiles
+    const int quarter = warp & 3, eg = warp >> 2;
     const int row = quarter * 32 + lane;
     const int m = rb * 128 + row;
     const int64_t pos = s.N - s.w + (m < M ? m % s.w : 0);   // causal limit of this row
     const float scale = kLog2e * rsqrtf((float)kHeadDim);
-    float rm = -INFINITY, rl = 0.f;
-    for (int i = 0; i < n_tiles; ++i) {
-      const int b = i & 1;
-      if (!mbar_wait_bounded(&sm.tfull[b], (i >> 1) & 1, kTries)) { sm.err = 1; break; }
+    bool bad = false;
+    for (int i = eg; i < n_tiles; i += P1_NGRP) {
+      const int b = i % P1_NACC;
+      if (!bad && !mbar_wait_bounded(&sm.tfull[b], (i / P1_NACC) & 1, kTries)) { sm.err = 1; bad = true; }
       tc_fence_after();
-      const int64_t t0 = t_begin + (int64_t)i * P1_TN + half * 128;
-      const uint32_t taddr = tmem + b * P1_TN + half * 128 + ((uint32_t)(quarter * 32) << 16);
-      // every token of this half-tile is a real token before the window, which every window row
-      // sees: no mask needed (warp-uniform)
-      const bool plain = t0 + 128 <= t_end && t0 + 128 <= s.N - s.w + 1;
+      const int64_t t0 = t_begin + (int64_t)i * P1_TN;
+      const uint32_t taddr = tmem + b * P1_TN + ((uint32_t)(quarter * 32) << 16);
+      // every token of this tile is a real token before the window, which every window row sees:
+      // no mask needed (warp-uniform)
+      const bool plain = t0 + P1_TN <= t_end && t0 + P1_TN <= s.N - s.w + 1;
 #pragma unroll
-      for (int cb = 0; cb < 4; ++cb) {
+      for (int cb = 0; cb < P1_TN / 32; ++cb) {
         float v[32];
         tmem_ld32(taddr + cb * 32, v);
-        if (plain) {
-          float cm = v[0];
-#pragma unroll
-          for (int jj = 1; jj < 32; ++jj) cm = fmaxf(cm, v[jj]);
-          const float nm = fmaxf(rm, cm * scale);   // scale > 0: max commutes with scaling
-          float sum = 0.f;
-#pragma unroll
-          for (int jj = 0; jj < 32; ++jj) sum += fast_exp2(fmaf(v[jj], scale, -nm));
-          rl = rl * fast_exp2(rm - nm) + sum;
-          rm = nm;
-        } else {
-          float cm = -INFINITY;
+        if (!plain) {
 #pragma unroll
           for (int jj = 0; jj < 32; ++jj) {
             const int64_t t = t0 + cb * 32 + jj;
-            v[jj] = (t < t_end && t <= pos) ? v[jj] * scale : -INFINITY;
-            cm = fmaxf(cm, v[jj]);
+            if (!(t < t_end && t <= pos)) v[jj] = -INFINITY;
           }
-          const float nm = fmaxf(rm, cm);
-          const float ref = nm == -INFINITY ? 0.f : nm;
-          float sum = 0.f;
-#pragma unroll
-          for (int jj = 0; jj < 32; ++jj) sum += fast_exp2(v[jj] - ref);
-          rl = rl * fast_exp2(rm - ref) + sum;
-          rm = nm;
         }
+        // max as a tree, sums in four interleaved partials (short dependency chains)
+        float mx[8];
+#pragma unroll
+        for (int q = 0; q < 8; ++q) mx[q] = fmaxf(fmaxf(v[4 * q], v[4 * q + 1]), fmaxf(v[4 * q + 2], v[4 * q + 3]));
+#pragma unroll
+        for (int q = 0; q < 4; ++q) mx[q] = fmaxf(mx[q], mx[q + 4]);
+        const float cm = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
+        const float nm = fmaxf(rm, cm * scale);    // scale > 0: max commutes with scaling
+        const float ref = nm == -INFINITY ? 0.f : nm;
+        float part[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int jj = 0; jj < 32; ++jj) part[jj & 3] += fast_exp2(fmaf(v[jj], scale, -ref));
+        rl = rl * fast_exp2(rm - ref) + ((part[0] + part[1]) + (part[2] + part[3]));
+        rm = nm;
       }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&sm.tempty[b]);
     }
-    sm.m[half][row] = rm;
-    sm.l[half][row] = rl;
   }
   tc_fence_before();
+  __syncthreads();
+  // every copy and product has landed: the group partials go through the idle key stages
+  float* gm = reinterpret_cast<float*>(kst);            // [P1_NGRP][128] maxima
+  float* gl = gm + P1_NGRP * 128;                       // [P1_NGRP][128] sums
+  if (warp < P1_EPI) {
+    gm[(warp >> 2) * 128 + (warp & 3) * 32 + lane] = rm;
+    gl[(warp >> 2) * 128 + (warp & 3) * 32 + lane] = rl;
+  }
   __syncthreads();
   if (tid < 128) {
     const int m = rb * 128 + tid;
     if (m < M) {
-      const float ma = sm.m[0][tid], mb = sm.m[1][tid];
-      const float mx = fmaxf(ma, mb);
+      float mx = -INFINITY;
+#pragma unroll
+      for (int e = 0; e < P1_NGRP; ++e) mx = fmaxf(mx, gm[e * 128 + tid]);
       float l = 0.f;
       if (mx != -INFINITY) {
-        if (ma != -INFINITY) l += sm.l[0][tid] * exp2f(ma - mx);
-        if (mb != -INFINITY) l += sm.l[1][tid] * exp2f(mb - mx);
+#pragma unroll
+        for (int e = 0; e < P1_NGRP; ++e)
+          if (gm[e * 128 + tid] != -INFINITY) l += gl[e * 128 + tid] * exp2f(gm[e * 128 + tid] - mx);
       }
       stats[((bl * s.G + g) * M + m) * n_chunks + blockIdx.x] = make_float2(mx, l);
     }
@@ -186,14 +192,16 @@ salience_stats_tc_kernel(const __grid_constant__ CUtensorMap tk, const __nv_bflo
 }
 
 // ------------------------------------------------------------------------------- pass 2
-constexpr int P2_EPI = 4;
+constexpr int P2_NGRP = 2;              // epilogue groups of four warps (tiles round-robin)
+constexpr int P2_EPI = 4 * P2_NGRP;
 constexpr int P2_THREADS = (P2_EPI + 2) * 32;
+constexpr int P2_NACC = 4;              // TMEM accumulator slots (npad <= 128: 4 x 128 columns)
 constexpr int P2_TM = 128;              // tokens per tile (MMA M)
-constexpr int P2_ST = 3;
+constexpr int P2_ST = 5;                // key stages (<= 224 KB with a 256-row window block)
 constexpr int P2_K = P2_TM * 256;       // 128 tokens x 128 bf16
 
 struct P2Smem {
-  uint64_t full[P2_ST], empty[P2_ST], tfull[2], tempty[2];
+  uint64_t full[P2_ST], empty[P2_ST], tfull[P2_NACC], tempty[P2_NACC];
   uint32_t tmem;
   int err;
   alignas(16) float nlse[256];   // negated log2-sum-exp per window row (-inf for padding rows)
@@ -220,6 +228,8 @@ salience_accum_tc_kernel(const __grid_constant__ CUtensorMap tk, const __nv_bflo
   const int64_t t_end = min(s.n_coded, t_begin + chunk2);
   if (t_begin >= t_end) return;
   const int nt = (int)((t_end - t_begin + P2_TM - 1) / P2_TM);
+  // accumulators of npad columns: four of 128 columns when npad <= 128, else two of 256
+  const int acc_cols = npad <= 128 ? 128 : 256, nacc = 512 / acc_cols;
 
   if (warp < P2_EPI) {
     // window rows of head g (swizzled K-major) and their negated lse
@@ -248,7 +258,7 @@ salience_accum_tc_kernel(const __grid_constant__ CUtensorMap tk, const __nv_bflo
   }
   if (warp == P2_EPI + 1 && lane == 0) {
     for (int i = 0; i < P2_ST; ++i) { mbar_init(&sm.full[i], 1); mbar_init(&sm.empty[i], 1); }
-    for (int i = 0; i < 2; ++i) { mbar_init(&sm.tfull[i], 1); mbar_init(&sm.tempty[i], P2_EPI); }
+    for (int i = 0; i < P2_NACC; ++i) { mbar_init(&sm.tfull[i], 1); mbar_init(&sm.tempty[i], 4); }
     sm.err = 0;
     fence_mbar_init();
   }
@@ -277,16 +287,16 @@ salience_accum_tc_kernel(const __grid_constant__ CUtensorMap tk, const __nv_bflo
       const uint32_t idesc = idesc_bf16_f32(P2_TM, npad);
       const uint32_t qa = smem_addr(qb);
       for (int i = 0; i < nt; ++i) {
-        const int st = i % P2_ST, b = i & 1;
+        const int st = i % P2_ST, b = i % nacc;
         if (!mbar_wait_bounded(&sm.full[st], (i / P2_ST) & 1, kTries) ||
-            !mbar_wait_bounded(&sm.tempty[b], ((i >> 1) & 1) ^ 1, kTries)) { sm.err = 1; break; }
+            !mbar_wait_bounded(&sm.tempty[b], ((i / nacc) & 1) ^ 1, kTries)) { sm.err = 1; break; }
         tc_fence_after();
         const uint32_t ka = smem_addr(kst + st * P2_K);
 #pragma unroll
         for (int ks = 0; ks < kHeadDim / 16; ++ks) {
           const uint32_t offk = (ks >> 2) * (P2_K / 2) + (ks & 3) * 32;   // K panel: 128 rows
           const uint32_t offq = (ks >> 2) * (npad * 128) + (ks & 3) * 32; // Q panel: npad rows
-          tc_mma_bf16(tmem + b * 256, sdesc_sw128(ka + offk), sdesc_sw128(qa + offq), idesc, ks > 0);
+          tc_mma_bf16(tmem + b * acc_cols, sdesc_sw128(ka + offk), sdesc_sw128(qa + offq), idesc, ks > 0);
         }
         tc_commit(&sm.empty[st]);
         tc_commit(&sm.tfull[b]);
@@ -295,12 +305,15 @@ salience_accum_tc_kernel(const __grid_constant__ CUtensorMap tk, const __nv_bflo
   } else {                                            // epilogue: one token per thread
     const float scale = kLog2e * rsqrtf((float)kHeadDim);
     float* out = raw_g + (bl * s.G + g) * s.n_coded;
-    for (int i = 0; i < nt; ++i) {
-      const int b = i & 1;
-      if (!mbar_wait_bounded(&sm.tfull[b], (i >> 1) & 1, kTries)) { sm.err = 1; break; }
+    const int eg = warp >> 2, row = tid & (P2_TM - 1);   // group eg takes tiles eg, eg + P2_NGRP, ...
+    bool bad = false;
+    for (int i = eg; i < nt; i += P2_NGRP) {
+      const int b = i % nacc;
+      if (!bad && !mbar_wait_bounded(&sm.tfull[b], (i / nacc) & 1, kTries)) { sm.err = 1; bad = true; }
       tc_fence_after();
-      const uint32_t taddr = tmem + b * 256 + ((uint32_t)(warp * 32) << 16);
-      float sum = 0.f;
+      const uint32_t taddr = tmem + b * acc_cols + ((uint32_t)((warp & 3) * 32) << 16);
+      // four partial sums in a fixed order (deterministic), so the adds do not form one chain
+      float part[4] = {0.f, 0.f, 0.f, 0.f};
       for (int cb = 0; cb < npad; cb += 32) {
         float v[32];
         tmem_ld32(taddr + cb, v);
@@ -308,17 +321,17 @@ salience_accum_tc_kernel(const __grid_constant__ CUtensorMap tk, const __nv_bflo
 #pragma unroll
         for (int q4 = 0; q4 < 8; ++q4) {
           const float4 n = nl[q4];
-          sum += fast_exp2(fmaf(v[4 * q4 + 0], scale, n.x));
-          sum += fast_exp2(fmaf(v[4 * q4 + 1], scale, n.y));
-          sum += fast_exp2(fmaf(v[4 * q4 + 2], scale, n.z));
-          sum += fast_exp2(fmaf(v[4 * q4 + 3], scale, n.w));
+          part[0] += fast_exp2(fmaf(v[4 * q4 + 0], scale, n.x));
+          part[1] += fast_exp2(fmaf(v[4 * q4 + 1], scale, n.y));
+          part[2] += fast_exp2(fmaf(v[4 * q4 + 2], scale, n.z));
+          part[3] += fast_exp2(fmaf(v[4 * q4 + 3], scale, n.w));
         }
       }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&sm.tempty[b]);
-      const int64_t t = t_begin + (int64_t)i * P2_TM + tid;
-      if (t < t_end) out[t] = sum;
+      const int64_t t = t_begin + (int64_t)i * P2_TM + row;
+      if (t < t_end) out[t] = (part[0] + part[1]) + (part[2] + part[3]);
     }
   }
   tc_fence_before();
@@ -395,17 +408,17 @@ int launch_salience_tc(const Shape& s, const void* q_win, const void* k, float* 
   off = (off + 255) & ~size_t(255);
   float* raw = reinterpret_cast<float*>(static_cast<char*>(ws) + off);
   const uint64_t rows = (uint64_t)s.B * s.L * s.G * s.N;
-  CUtensorMap t256, t128;
-  if (!make_tmap_rows_bf16(&t256, k, rows, P1_TN) || !make_tmap_rows_bf16(&t128, k, rows, P2_TM)) return -1;
+  CUtensorMap tmap1, tmap2;   // boxes of P1_TN and P2_TM rows
+  if (!make_tmap_rows_bf16(&tmap1, k, rows, P1_TN) || !make_tmap_rows_bf16(&tmap2, k, rows, P2_TM)) return -1;
   const size_t smem1 = 1024 + P1_Q + P1_ST * P1_K + sizeof(P1Smem);
   cudaFuncSetAttribute(salience_stats_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem1);
   salience_stats_tc_kernel<<<dim3(p.n_chunks, s.G * p.n_rb, s.B * s.L), P1_THREADS, smem1, st>>>(
-      t256, (const __nv_bfloat16*)q_win, stats, dev_status, s, p.n_chunks, p.chunk, p.n_rb);
+      tmap1, (const __nv_bfloat16*)q_win, stats, dev_status, s, p.n_chunks, p.chunk, p.n_rb);
   const size_t qbytes = ((size_t)npad * 256 + 1023) & ~size_t(1023);
   const size_t smem2 = 1024 + P2_ST * P2_K + qbytes + sizeof(P2Smem);
   cudaFuncSetAttribute(salience_accum_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem2);
   salience_accum_tc_kernel<<<dim3(p.n_chunks2, s.G, s.B * s.L), P2_THREADS, smem2, st>>>(
-      t128, (const __nv_bfloat16*)q_win, stats, raw, dev_status, s, p.n_chunks, p.chunk2, npad);
+      tmap2, (const __nv_bfloat16*)q_win, stats, raw, dev_status, s, p.n_chunks, p.chunk2, npad);
   salience_pool_tc_kernel<<<dim3((unsigned)((s.n_coded + 255) / 256), s.B * s.L), 256, 0, st>>>(raw, sal_out, s);
   return 3;
 }
