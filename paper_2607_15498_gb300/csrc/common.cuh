@@ -57,6 +57,14 @@ __device__ __forceinline__ void load8_stream(const float* p, float (&f)[8]) {
 
 __device__ __forceinline__ int64_t pad8(int64_t n) { return (n + 7) & ~int64_t(7); }
 
+// Read-only 32-bit global load issued exactly where it is written (volatile: the compiler may not
+// sink it past later barriers), so its latency overlaps with the work that follows.
+__device__ __forceinline__ uint32_t ld_nc_early(const uint32_t* p) {
+  uint32_t v;
+  asm volatile("ld.global.nc.u32 %0, [%1];\n" : "=r"(v) : "l"(p));
+  return v;
+}
+
 }  // namespace vr
 
 namespace vr {

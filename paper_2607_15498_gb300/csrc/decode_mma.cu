@@ -182,12 +182,12 @@ __device__ __forceinline__ void rot_load(RotRegs& rr, const __nv_bfloat16* __res
 #pragma unroll
   for (int kc = 0; kc < kHeadDim / 16; ++kc) {
     const int i0 = kc * 16;
-    rr.a[kc][0] = __ldg(Uw + ((j0 + g8) * kHeadDim + i0 + 2 * c) / 2);
-    rr.a[kc][1] = __ldg(Uw + ((j0 + g8 + 8) * kHeadDim + i0 + 2 * c) / 2);
-    rr.a[kc][2] = __ldg(Uw + ((j0 + g8) * kHeadDim + i0 + 2 * c + 8) / 2);
-    rr.a[kc][3] = __ldg(Uw + ((j0 + g8 + 8) * kHeadDim + i0 + 2 * c + 8) / 2);
-    rr.bq[kc][0] = __ldg(qw + (i0 + 2 * c) / 2);
-    rr.bq[kc][1] = __ldg(qw + (i0 + 2 * c + 8) / 2);
+    rr.a[kc][0] = ld_nc_early(Uw + ((j0 + g8) * kHeadDim + i0 + 2 * c) / 2);
+    rr.a[kc][1] = ld_nc_early(Uw + ((j0 + g8 + 8) * kHeadDim + i0 + 2 * c) / 2);
+    rr.a[kc][2] = ld_nc_early(Uw + ((j0 + g8) * kHeadDim + i0 + 2 * c + 8) / 2);
+    rr.a[kc][3] = ld_nc_early(Uw + ((j0 + g8 + 8) * kHeadDim + i0 + 2 * c + 8) / 2);
+    rr.bq[kc][0] = ld_nc_early(qw + (i0 + 2 * c) / 2);
+    rr.bq[kc][1] = ld_nc_early(qw + (i0 + 2 * c + 8) / 2);
   }
 }
 

@@ -240,5 +240,6 @@ class PackedCache:
 
 
 def workspace(cfg: varrate_config, which_call: int, device="cuda") -> torch.Tensor:
+    """Device scratch for one kind of call (zero-filled; no call needs particular contents)."""
     n = varrate_workspace_bytes(cfg, which_call)
-    return torch.empty(max(n, 256), dtype=torch.uint8, device=device)
+    return torch.zeros(max(n, 256), dtype=torch.uint8, device=device)
