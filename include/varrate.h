@@ -176,10 +176,13 @@ varrate_status varrate_encode(const varrate_config* cfg, const void* q_win, cons
  *   tail_k/_v [B][G][n_tail][d] uncompressed tokens appended after the cache (may be NULL if
  *           n_tail == 0)
  *   out     [B][H][d]  dtype
- *   ws      at least varrate_workspace_bytes(cfg, VARRATE_CALL_DECODE) bytes; no contents
- *           required (in bf16 the call clears its per-(sequence, KV head) completion counters in
- *           the workspace on `stream` before its one kernel, so calls sharing a workspace must be
- *           ordered on one stream). */
+ *   ws      at least varrate_workspace_bytes(cfg, VARRATE_CALL_DECODE) bytes, zero-filled before
+ *           the first decode call that uses it. Its first 16 KiB hold per-(sequence, KV head)
+ *           completion counters that every call leaves at zero again; the rest is scratch that a
+ *           call writes before it reads. So one workspace serves any number of later decode calls
+ *           (any shape), provided they are ordered on one stream. A call that finds a counter
+ *           that is not zero raises VARRATE_ERR_CORRUPT in *dev_status: zero the workspace again
+ *           before its next use. */
 varrate_status varrate_decode_attn(const varrate_config* cfg, const varrate_packed* cache,
                                    const void* basis_k, const void* basis_v, const void* q,
                                    int32_t layer, const void* tail_k, const void* tail_v,
@@ -197,9 +200,9 @@ varrate_status varrate_decode_attn(const varrate_config* cfg, const varrate_pack
  *  - The first call on a device looks up the array's device address (once per device, for the
  *    current device); make that first call before any stream capture.
  *  - All calls share the one array: calls that overlap on the GPU (other streams, other host
- *    threads) race on it and must be serialised by the caller. No contents carry over that matter:
- *    every scratch element is written (the completion counters cleared on the stream) before it
- *    is read. */
+ *    threads) race on it and must be serialised by the caller. The array starts zero-filled; its
+ *    completion counters are left at zero by every call and the rest is written before it is
+ *    read, so no contents carry over that matter. */
 varrate_status varrate_decode_attn_noalloc(const varrate_config* cfg, const varrate_packed* cache,
                                            const void* basis_k, const void* basis_v, const void* q,
                                            int32_t layer, const void* tail_k, const void* tail_v,

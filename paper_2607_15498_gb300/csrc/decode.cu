@@ -364,16 +364,18 @@ size_t decode_ws_bytes(const Shape& s, int num_sms) {
   a += (size_t)s.B * s.G * S * group_pad(s.grp) * (kHeadDim + 2) * sizeof(float);
   const size_t m = decode_mma_part_bytes(s, num_sms);
   if (m > a) a = m;
-  return (a + 255) & ~size_t(255);
+  return kDecodeCounterBytes + ((a + 255) & ~size_t(255));
 }
 
 int launch_decode(const Shape& s, const varrate_packed& cache, const void* basis_k,
                   const void* basis_v, const void* q, int layer, const void* tail_k,
                   const void* tail_v, int n_tail, void* out, int32_t* dev_status, void* ws,
                   int num_sms, cudaStream_t st) {
+  int* seg_done = reinterpret_cast<int*>(ws);   // completion counters: the first kDecodeCounterBytes
+  ws = static_cast<char*>(ws) + kDecodeCounterBytes;
   if (decode_mma_supported(s, n_tail, num_sms))
     return launch_decode_mma(s, cache, basis_k, basis_v, q, layer, tail_k, tail_v, n_tail, out,
-                             dev_status, reinterpret_cast<float*>(ws), num_sms, st);
+                             dev_status, seg_done, reinterpret_cast<float*>(ws), num_sms, st);
   const int S = decode_splits(s, num_sms);
   float* qt = reinterpret_cast<float*>(ws);
   size_t a = (size_t)s.B * s.H * kHeadDim * sizeof(float);

@@ -25,9 +25,13 @@
 //   values   O~^T[j][head] += V[j][slot] * P^T[slot][head]      (P in bf16, <= 2^-9 relative per
 //            weight, transposed from the score fragments with movmatrix)
 // Partials (max, sum, o~[128]) per (segment, CTA) go to the workspace. The last CTA to finish a
-// segment (a per-segment counter in the workspace, zeroed before the launch) merges its partials,
-// adds the exact tail, rotates back with U_V^T (staged in the idle ring) and normalises, so one
-// launch does the whole step.
+// segment (a per-segment counter in the workspace, which that CTA sets back to zero for the next
+// call) merges its partials, adds the exact tail, rotates back with U_V^T (staged in the idle ring)
+// and normalises, so one launch does the whole step.
+//
+// Warps reconverge explicitly (__syncwarp) after lane-dependent code and before warp-wide
+// shuffles, votes and tensor-core fragments: left to itself a diverged warp reaching those
+// instructions was measured to lose thousands of cycles.
 #include <stddef.h>
 
 #include "common.cuh"
@@ -138,6 +142,7 @@ __device__ __forceinline__ bool issue_chunk(Prod& p, const SegSmem& sm, const __
     bulk_g2s_hint(stage_addr, (p.phase ? cV : cK) + sm.base[r] + t0 * r + (long long)j0 * tl, bytes, bar,
                   l2_evict_first_policy());
   }
+  __syncwarp();   // lane 0 branched off: reconverge before the next warp-wide instruction
   const int nj = (r + CH - 1) / CH;
   if (++p.jc == nj) {
     p.jc = 0;
@@ -275,6 +280,7 @@ __device__ bool combine_segment(CombSmem& cs, uint64_t* bar, uint32_t parity, co
     mbar_arrive_expect_tx(bar, kHeadDim * kHeadDim * 2);
     bulk_g2s(smem_addr(cs.us), Uv, kHeadDim * kHeadDim * 2, bar);
   }
+  __syncwarp();
   const float scale = kLog2e * rsqrtf((float)kHeadDim);
   if (n_tail) {                                                   // exact tail scores and maxima
     for (int i = tid; i < grp * kHeadDim; i += blockDim.x) cs.qrow[i / kHeadDim][i % kHeadDim] = __bfloat162float(q[i]);
@@ -342,6 +348,7 @@ __device__ bool combine_segment(CombSmem& cs, uint64_t* bar, uint32_t parity, co
   }
   *reinterpret_cast<float4*>(&cs.ot[h][4 * lane]) = acc;        // zero for padded heads
   if (!__syncthreads_and(mbar_wait_bounded(bar, parity, kWaitTries))) return false;
+  __syncwarp();
   // out^T[col][head] = sum_j U_V[j][col] o~[head][j]: warp w owns columns 16w .. 16w + 15
   {
     float d[4] = {0.f, 0.f, 0.f, 0.f};
@@ -400,6 +407,9 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
   const int g8 = lane >> 2, c = lane & 3;
   const int C = gridDim.x, cta = blockIdx.x;
 
+  // the next grid in the stream may be scheduled now: it only starts on SMs this grid has left,
+  // and waits (griddepcontrol.wait) for this grid to finish before it reads anything
+  pdl_trigger();
   // self-contained setup first (it may overlap the tail of the preceding grid)
   // the ring only ever holds finite coefficients or zeros
   for (int i = tid; i < NW * ST * STAGE / 16; i += blockDim.x)
@@ -422,6 +432,7 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
   // Cost line: sequence b holds G segments of kSegCost + W_b elements each (W_b > 0), the set-up
   // allowance first. segP = exclusive prefix over sequences (B <= 64: two per lane).
   if (warp == 0) {
+    __syncwarp();   // lanes left the loads above apart: reconverge before the shuffles
     const int e0 = 2 * lane, e1 = 2 * lane + 1;
     const long long v0 = (e0 < s.B && segW[e0]) ? (segW[e0] + kSegCost) * s.G : 0;
     const long long v1 = (e1 < s.B && segW[e1]) ? (segW[e1] + kSegCost) * s.G : 0;
@@ -482,6 +493,7 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
       }
       __syncthreads();
       if (warp == 0) {   // inclusive scan of it_pref[1 .. 129], 5 entries per lane
+        __syncwarp();
         constexpr int kPer = (kMaxR + 1 + 31) / 32;
         int v[kPer], acc = 0;
 #pragma unroll
@@ -528,6 +540,7 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
                         &bars[(n_issued + i) % ST], total, lane)) ++n_pending;
       int c0, c1;   // the CTAs that share this segment (their partials are merged by the last one)
       seg_cta_range(cuts, C, P, W, c0, c1);
+      __syncwarp();
       rot_compute(sm, rr, s.grp, warp, lane);
       __syncthreads();
       build_qfrag(sm, tid);
@@ -695,6 +708,7 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
       }
 
       // ---- merge the warps of this CTA for this segment
+      __syncwarp();
 #pragma unroll
       for (int e = 0; e < 2; ++e)
 #pragma unroll
@@ -742,7 +756,11 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
       __syncthreads();
       if (tid == 0) {
         __threadfence();
-        last_cta = atomicAdd(&seg_done[seg], 1) == c1 - c0;
+        const unsigned done = (unsigned)atomicAdd(&seg_done[seg], 1);
+        last_cta = done == (unsigned)(c1 - c0);
+        // every CTA of the segment has counted: zero again for the next call on this workspace
+        if (last_cta) seg_done[seg] = 0;
+        else if (done > (unsigned)(c1 - c0)) raise_status(dev_status, VARRATE_ERR_CORRUPT);
       }
       __syncthreads();
       if (last_cta) {
@@ -785,30 +803,30 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
       ++n_comb;
     }
   if (timed_out && lane == 0) raise_status(dev_status, VARRATE_ERR_TIMEOUT);
-  pdl_trigger();
 }
 
 }  // namespace
 
 size_t decode_mma_smem_bytes() { return (size_t)NW * ST * STAGE + sizeof(SegSmem); }
 
-// partials, then one completion counter per (sequence, head) segment
+// partials: one slot per (segment, CTA) pair a CTA can meet (the counters live apart, see kernels.h)
 size_t decode_mma_part_bytes(const Shape& s, int num_sms) {
   const size_t p = (size_t)(num_sms + (size_t)s.B * s.G) * kHeadsPad * kPartStride * sizeof(float);
-  return ((p + 255) & ~size_t(255)) + (size_t)s.B * s.G * sizeof(int);
+  return (p + 255) & ~size_t(255);
 }
 
 bool decode_mma_supported(const Shape& s, int n_tail, int num_sms) {
   // the cost line (at most B G cap elements) times the grid size must stay below 2^62
   const unsigned long long line = (unsigned long long)s.B * s.G * ((unsigned long long)s.cap + kSegCost);
-  return s.dtype == VARRATE_BF16 && s.B <= 64 && n_tail <= 64 && num_sms >= 1 &&
-         num_sms <= kMaxCtas && line <= (1ull << 62) / (unsigned long long)num_sms;
+  return s.dtype == VARRATE_BF16 && s.B <= 64 && (long long)s.B * s.G <= kDecodeMaxSegs &&
+         n_tail <= 64 && num_sms >= 1 && num_sms <= kMaxCtas &&
+         line <= (1ull << 62) / (unsigned long long)num_sms;
 }
 
 int launch_decode_mma(const Shape& s, const varrate_packed& c, const void* basis_k,
                       const void* basis_v, const void* q, int layer, const void* tail_k,
-                      const void* tail_v, int n_tail, void* out, int32_t* dev_status, float* part,
-                      int num_sms, cudaStream_t st) {
+                      const void* tail_v, int n_tail, void* out, int32_t* dev_status, int* seg_done,
+                      float* part, int num_sms, cudaStream_t st) {
   const size_t smem = decode_mma_smem_bytes();
   cudaFuncSetAttribute(decode_mma_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   // the grid may be scheduled while its predecessor drains (programmatic dependent launch); it
@@ -823,9 +841,6 @@ int launch_decode_mma(const Shape& s, const varrate_packed& c, const void* basis
   lc.stream = st;
   lc.attrs = pdl;
   lc.numAttrs = 1;
-  const size_t pbytes = ((size_t)(num_sms + (size_t)s.B * s.G) * kHeadsPad * kPartStride * sizeof(float) + 255) & ~size_t(255);
-  int* seg_done = reinterpret_cast<int*>(reinterpret_cast<char*>(part) + pbytes);
-  cudaMemsetAsync(seg_done, 0, (size_t)s.B * s.G * sizeof(int), st);
   cudaLaunchKernelEx(&lc, decode_mma_kernel, (const __nv_bfloat16*)c.coef, (const int32_t*)c.bucket_count,
                      (const int64_t*)c.bucket_base, (const __nv_bfloat16*)basis_k,
                      (const __nv_bfloat16*)basis_v, (const __nv_bfloat16*)q,

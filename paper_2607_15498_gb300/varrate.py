@@ -240,6 +240,7 @@ class PackedCache:
 
 
 def workspace(cfg: varrate_config, which_call: int, device="cuda") -> torch.Tensor:
-    """Device scratch for one kind of call (zero-filled; no call needs particular contents)."""
+    """Device scratch for one kind of call, zero-filled (decode needs zeros before its first call
+    and leaves its completion counters at zero after each one)."""
     n = varrate_workspace_bytes(cfg, which_call)
     return torch.zeros(max(n, 256), dtype=torch.uint8, device=device)

@@ -227,6 +227,41 @@ def test_decode_floor_binds(inputs):
     _decode_check(CASES["qwen_g7"], inputs["qwen_g7"], budget_frac=0.10, n_steps=2)
 
 
+def _decode_with_ws(cfg, packed, bk, bv, q, layer, ws):
+    out = torch.empty_like(q, device="cuda")
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    V.check(V.varrate_decode_attn(cfg, packed, bk.cuda(), bv.cuda(), q.cuda(), layer, None, None, 0,
+                                  out, status, ws), "varrate_decode_attn")
+    torch.cuda.synchronize()
+    return f64(out), int(status.item())
+
+
+def test_decode_workspace_reuse_and_counter_check(inputs):
+    """One zero-filled workspace serves decode calls of different shapes in any order: every call
+    leaves the completion counters (the workspace's first 16 KiB) at zero and its outputs equal
+    those of a call on a fresh workspace. A counter that is not zero is reported as corrupt."""
+    runs = []
+    for name in ("llama_ragged", "qwen_g7"):
+        wl = CASES[name]
+        k, v, qw, bk, bv = inputs[name]
+        cfg = cfg_for(wl)
+        r = gpu_encode(cfg, k, v, qw, bk, bv)
+        runs.append((cfg, r["packed"], bk, bv, synth.stack_decode_queries(wl, 0, 1)[0]))
+    ref = [gpu_decode(cfg, p, bk, bv, q, 0)[0] for (cfg, p, bk, bv, q) in runs]
+    n = max(V.varrate_workspace_bytes(run[0], V.CALL_DECODE) for run in runs)
+    ws = torch.zeros(n, dtype=torch.uint8, device="cuda")
+    for _ in range(3):
+        for i, (cfg, p, bk, bv, q) in enumerate(runs):
+            out, st = _decode_with_ws(cfg, p, bk, bv, q, 0, ws)
+            assert st == V.OK
+            np.testing.assert_array_equal(out, ref[i])
+    assert int(torch.count_nonzero(ws[:16384])) == 0
+    ws[:16384].fill_(0x7F)
+    cfg, p, bk, bv, q = runs[0]
+    _, st = _decode_with_ws(cfg, p, bk, bv, q, 0, ws)
+    assert st == V.ERR_CORRUPT
+
+
 def test_budget_one_matches_uncompressed_attention():
     wl = synth.workload("tiny", n_ctx=1500, budget_frac=1.0)
     k, v, qw, bk, bv = synth.stack_inputs(wl)
