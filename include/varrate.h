@@ -9,8 +9,9 @@
  *
  * Conventions shared by every entry point
  *  - Every tensor argument is a caller-owned DEVICE pointer (CUDA global memory), row-major and
- *    densely packed in the layout stated next to it. The library never allocates or frees device
- *    memory and keeps no state between calls (reentrant).
+ *    densely packed in the layout stated next to it, and 16-byte aligned (as cudaMalloc and
+ *    PyTorch allocations are); a misaligned pointer is VARRATE_ERR_ARG. The library never
+ *    allocates or frees device memory and keeps no state between calls (reentrant).
  *  - `stream` is a cudaStream_t passed as void* (NULL = the legacy default stream). Every call
  *    only enqueues work on `stream` and returns without synchronising.
  *  - The return value reports what the host can see: bad arguments (VARRATE_ERR_ARG), a workspace

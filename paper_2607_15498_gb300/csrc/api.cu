@@ -1,5 +1,6 @@
 // C ABI of the VarRate hot path (declared in include/varrate.h): argument validation, workspace
 // carving and kernel launches. No device memory is allocated here.
+#include <initializer_list>
 #include <math.h>
 #include <stdint.h>
 
@@ -89,9 +90,18 @@ varrate_status launched() {
   return cudaGetLastError() == cudaSuccess ? VARRATE_OK : VARRATE_ERR_CUDA;
 }
 
+// Every device pointer must be 16-byte aligned: the kernels move data with 16-byte vector loads,
+// 1-D bulk copies and TMA tiles, which fault on misaligned addresses. NULL passes.
+bool aligned16(std::initializer_list<const void*> ps) {
+  for (const void* p : ps)
+    if ((reinterpret_cast<uintptr_t>(p) & 15u) != 0) return false;
+  return true;
+}
+
 bool packed_ok(const varrate_config* c, const varrate_packed* p) {
   return p && p->coef && p->bucket_count && p->bucket_base && p->perm && p->pos && p->ranks &&
-         p->cap_elems >= cap_elems(c) && (p->cap_elems % 8) == 0;
+         p->cap_elems >= cap_elems(c) && (p->cap_elems % 8) == 0 &&
+         aligned16({p->coef, p->bucket_count, p->bucket_base, p->perm, p->pos, p->ranks});
 }
 
 }  // namespace
@@ -135,6 +145,7 @@ varrate_status varrate_salience(const varrate_config* cfg, const void* q_win, co
   const bool empty = cfg->n_ctx == cfg->window;   // no coded token: nothing to score
   if (!empty && (!q_win || !k || !sal_out)) return VARRATE_ERR_ARG;
   if (cfg->mode == VARRATE_UNIFORM) return VARRATE_ERR_ARG;
+  if (!aligned16({q_win, k, sal_out, ws})) return VARRATE_ERR_ARG;
   const size_t need = ws_bytes(cfg, VARRATE_CALL_SALIENCE);
   if (ws_bytes_ < need || (need > 0 && ws == nullptr)) return VARRATE_ERR_WORKSPACE;
   const Shape s = make_shape(cfg, cap_elems(cfg));
@@ -149,6 +160,7 @@ varrate_status varrate_allocate(const varrate_config* cfg, const float* sal, uin
   if (st != VARRATE_OK) return st;
   if (!ranks || (cfg->mode == VARRATE_SALIENCE && !sal && cfg->n_ctx > cfg->window))
     return VARRATE_ERR_ARG;
+  if (!aligned16({sal, ranks, realized_sum, dev_status})) return VARRATE_ERR_ARG;
   const Shape s = make_shape(cfg, cap_elems(cfg));
   vr::launch_allocate(s, sal, ranks, realized_sum, dev_status, (cudaStream_t)stream);
   return launched();
@@ -161,6 +173,7 @@ varrate_status varrate_pack(const varrate_config* cfg, const void* k, const void
   varrate_status st = check(cfg);
   if (st != VARRATE_OK) return st;
   if (!k || !v || !basis_k || !basis_v || !packed_ok(cfg, out)) return VARRATE_ERR_ARG;
+  if (!aligned16({k, v, basis_k, basis_v, dev_status})) return VARRATE_ERR_ARG;
   const Shape s = make_shape(cfg, out->cap_elems);
   if (!vr::pack_ready(s, k, v)) return VARRATE_ERR_CUDA;   // before anything is enqueued
   if (vr::launch_pack(s, k, v, basis_k, basis_v, *out, dev_status, num_sms(), (cudaStream_t)stream) < 0)
@@ -176,6 +189,8 @@ varrate_status varrate_encode(const varrate_config* cfg, const void* q_win, cons
   if (st != VARRATE_OK) return st;
   if (!k || !v || !basis_k || !basis_v || !packed_ok(cfg, out)) return VARRATE_ERR_ARG;
   if (cfg->mode == VARRATE_SALIENCE && !q_win && cfg->n_ctx > cfg->window) return VARRATE_ERR_ARG;
+  if (!aligned16({q_win, k, v, basis_k, basis_v, sal_out, realized_sum, dev_status, ws}))
+    return VARRATE_ERR_ARG;
   const size_t need = ws_bytes(cfg, VARRATE_CALL_ENCODE);
   if (ws_bytes_ < need || ws == nullptr) return VARRATE_ERR_WORKSPACE;
   const Shape s = make_shape(cfg, out->cap_elems);
@@ -206,6 +221,7 @@ varrate_status varrate_decode_attn(const varrate_config* cfg, const varrate_pack
   if (layer < 0 || layer >= cfg->n_layers || n_tail < 0) return VARRATE_ERR_ARG;
   if (n_tail > 4096) return VARRATE_ERR_UNSUPPORTED;
   if (n_tail > 0 && (!tail_k || !tail_v)) return VARRATE_ERR_ARG;
+  if (!aligned16({basis_k, basis_v, q, tail_k, tail_v, out, dev_status, ws})) return VARRATE_ERR_ARG;
   const size_t need = ws_bytes(cfg, VARRATE_CALL_DECODE);
   if (ws_bytes_ < need || ws == nullptr) return VARRATE_ERR_WORKSPACE;
   const Shape s = make_shape(cfg, cache->cap_elems);

@@ -233,21 +233,15 @@ __device__ __forceinline__ long long cut_at(long long T, long long c, int C) {
   return (long long)(((unsigned long long)T * (unsigned long long)c) / (unsigned long long)C);
 }
 
-// CTAs whose cost range [cuts[c], cuts[c + 1]) meets [P, P + W): c0..c1 (W > 0).
-__device__ __forceinline__ void seg_cta_range(const long long* cuts, int C, long long P, long long W,
-                                              int& c0, int& c1) {
-  int lo = 0, hi = C - 1;   // first c with cuts[c + 1] > P (cuts[C] = T > P)
-  while (lo < hi) {
-    const int mid = (lo + hi) >> 1;
-    if (cuts[mid + 1] > P) hi = mid; else lo = mid + 1;
-  }
-  c0 = lo;
-  lo = c0; hi = C;          // first c with cuts[c] > P + W - 1, or C
-  while (lo < hi) {
-    const int mid = (lo + hi) >> 1;
-    if (cuts[mid] > P + W - 1) hi = mid; else lo = mid + 1;
-  }
-  c1 = lo - 1;
+// CTAs whose cost range [cuts[c], cuts[c + 1]) meets [P, P + W): c0..c1 (W > 0, P + W <= T).
+// With cuts[c] = floor(T c / C): cuts[c + 1] > P  <=>  c + 1 >= ceil((P + 1) C / T), and
+// cuts[c] > P + W - 1  <=>  c >= ceil((P + W) C / T); both products stay below T C < 2^62.
+__device__ __forceinline__ void seg_cta_range(long long T, int C, long long P, long long W, int& c0,
+                                              int& c1) {
+  const unsigned long long t = (unsigned long long)T, cc = (unsigned long long)C;
+  c0 = (int)(((unsigned long long)(P + 1) * cc + t - 1) / t) - 1;
+  const unsigned long long f = ((unsigned long long)(P + W) * cc + t - 1) / t;
+  c1 = (int)(f < cc ? f : cc) - 1;
 }
 
 constexpr int kMaxCtas = 1024;   // grid size bound (64-bit cost-line arithmetic)
@@ -539,7 +533,7 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
         if (issue_chunk(pr, sm, cK, cV, ring_w + ((n_issued + i) % ST) * STAGE,
                         &bars[(n_issued + i) % ST], total, lane)) ++n_pending;
       int c0, c1;   // the CTAs that share this segment (their partials are merged by the last one)
-      seg_cta_range(cuts, C, P, W, c0, c1);
+      seg_cta_range(T, C, P, W, c0, c1);
       __syncwarp();
       rot_compute(sm, rr, s.grp, warp, lane);
       __syncthreads();

@@ -20,6 +20,9 @@ def declared_functions():
     return sorted(set(re.findall(r"\b(varrate_\w+)\s*\(", text)))
 
 
+A = 1 << 12   # a 16-byte aligned fake device pointer (never dereferenced: host-side checks only)
+
+
 def test_header_declares_the_hot_path():
     names = declared_functions()
     for must in ("varrate_encode", "varrate_allocate", "varrate_pack", "varrate_decode_attn",
@@ -110,19 +113,39 @@ def test_small_workspace_and_bad_layer_rejected_on_host(vlib):
     cfg = vlib.make_config(2, 1, 4, 2048, dtype=vlib.F32)
     L = vlib.lib()
     cap = vlib.varrate_packed_cap_elems(cfg)
-    p = vlib.varrate_packed(1, 1, 1, 1, 1, 1, cap)
-    assert L.varrate_decode_attn(vlib.ctypes.byref(cfg), vlib.ctypes.byref(p), 1, 1, 1, 2, None,
-                                 None, 0, 1, None, 1, 1 << 40, None) == vlib.ERR_ARG
-    assert L.varrate_decode_attn(vlib.ctypes.byref(cfg), vlib.ctypes.byref(p), 1, 1, 1, 0, None,
-                                 None, 0, 1, None, 1, 16, None) == vlib.ERR_WORKSPACE
-    assert L.varrate_decode_attn(vlib.ctypes.byref(cfg), vlib.ctypes.byref(p), 1, 1, 1, 0, None,
-                                 None, 5000, 1, None, 1, 1 << 40, None) == vlib.ERR_UNSUPPORTED
+    p = vlib.varrate_packed(A, A, A, A, A, A, cap)
+    assert L.varrate_decode_attn(vlib.ctypes.byref(cfg), vlib.ctypes.byref(p), A, A, A, 2, None,
+                                 None, 0, A, None, A, 1 << 40, None) == vlib.ERR_ARG
+    assert L.varrate_decode_attn(vlib.ctypes.byref(cfg), vlib.ctypes.byref(p), A, A, A, 0, None,
+                                 None, 0, A, None, A, 16, None) == vlib.ERR_WORKSPACE
+    assert L.varrate_decode_attn(vlib.ctypes.byref(cfg), vlib.ctypes.byref(p), A, A, A, 0, None,
+                                 None, 5000, A, None, A, 1 << 40, None) == vlib.ERR_UNSUPPORTED
     p.cap_elems = cap - 8
-    assert L.varrate_decode_attn(vlib.ctypes.byref(cfg), vlib.ctypes.byref(p), 1, 1, 1, 0, None,
-                                 None, 0, 1, None, 1, 1 << 40, None) == vlib.ERR_ARG
-    assert L.varrate_encode(vlib.ctypes.byref(cfg), 1, 1, 1, 1, 1, None,
-                            vlib.ctypes.byref(vlib.varrate_packed(1, 1, 1, 1, 1, 1, cap)), None,
-                            None, 1, 8, None) == vlib.ERR_WORKSPACE
+    assert L.varrate_decode_attn(vlib.ctypes.byref(cfg), vlib.ctypes.byref(p), A, A, A, 0, None,
+                                 None, 0, A, None, A, 1 << 40, None) == vlib.ERR_ARG
+    assert L.varrate_encode(vlib.ctypes.byref(cfg), A, A, A, A, A, None,
+                            vlib.ctypes.byref(vlib.varrate_packed(A, A, A, A, A, A, cap)), None,
+                            None, A, 8, None) == vlib.ERR_WORKSPACE
+
+
+def test_misaligned_pointers_rejected_on_host(vlib):
+    """Bulk copies and TMA need 16-byte aligned addresses: a misaligned device pointer is an
+    argument error found on the host, before anything is enqueued."""
+    cfg = vlib.make_config(2, 1, 4, 2048, dtype=vlib.BF16)
+    L = vlib.lib()
+    cap = vlib.varrate_packed_cap_elems(cfg)
+    p = vlib.varrate_packed(A, A, A, A, A, A, cap)
+    args = [A, A, A]                       # basis_k, basis_v, q
+    for i in range(3):
+        bad = list(args)
+        bad[i] = A + 2
+        assert L.varrate_decode_attn(vlib.ctypes.byref(cfg), vlib.ctypes.byref(p), *bad, 0, None,
+                                     None, 0, A, None, A, 1 << 40, None) == vlib.ERR_ARG
+    q = vlib.varrate_packed(A + 8, A, A, A, A, A, cap)
+    assert L.varrate_decode_attn(vlib.ctypes.byref(cfg), vlib.ctypes.byref(q), A, A, A, 0, None,
+                                 None, 0, A, None, A, 1 << 40, None) == vlib.ERR_ARG
+    assert L.varrate_pack(vlib.ctypes.byref(cfg), A + 4, A, A, A, vlib.ctypes.byref(p), None, None,
+                          0, None) == vlib.ERR_ARG
 
 
 def test_binding_fails_loudly_without_library(tmp_path, monkeypatch):
