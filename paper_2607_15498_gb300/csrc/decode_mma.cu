@@ -345,7 +345,9 @@ __device__ bool combine_segment(CombSmem& cs, uint64_t* bar, uint32_t parity, co
   __syncwarp();
   // out^T[col][head] = sum_j U_V[j][col] o~[head][j]: warp w owns columns 16w .. 16w + 15
   {
-    float d[4] = {0.f, 0.f, 0.f, 0.f};
+    // four independent accumulators (hi / lo part of o~, even / odd k-step) keep the chain of
+    // dependent MMAs four deep instead of sixteen
+    float d[4][4] = {};
     const int col0 = warp * 16;
 #pragma unroll
     for (int ks = 0; ks < kHeadDim / 16; ++ks) {
@@ -357,14 +359,14 @@ __device__ bool combine_segment(CombSmem& cs, uint64_t* bar, uint32_t parity, co
       uint32_t h0, l0, h1, l1;
       split_bf16(cs.ot[g8][jb], cs.ot[g8][jb + 1], h0, l0);
       split_bf16(cs.ot[g8][jb + 8], cs.ot[g8][jb + 9], h1, l1);
-      mma_bf16_16816(d, a, h0, h1);
-      mma_bf16_16816(d, a, l0, l1);
+      mma_bf16_16816(d[ks & 1], a, h0, h1);
+      mma_bf16_16816(d[2 + (ks & 1)], a, l0, l1);
     }
 #pragma unroll
     for (int e = 0; e < 4; ++e) {
       const int col = col0 + g8 + (e >> 1) * 8, hh = 2 * c + (e & 1);
       if (hh < grp) {
-        float y = d[e];
+        float y = (d[0][e] + d[1][e]) + (d[2][e] + d[3][e]);
         for (int t = 0; t < n_tail; ++t)
           y = fmaf(cs.tsc[hh][t], __bfloat162float(tail_v[(long long)t * kHeadDim + col]), y);
         out[(long long)hh * kHeadDim + col] = __float2bfloat16_rn(y / cs.hl[hh]);
@@ -753,12 +755,15 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
         const unsigned done = (unsigned)atomicAdd(&seg_done[seg], 1);
         last_cta = done == (unsigned)(c1 - c0);
         // every CTA of the segment has counted: zero again for the next call on this workspace
-        if (last_cta) seg_done[seg] = 0;
-        else if (done > (unsigned)(c1 - c0)) raise_status(dev_status, VARRATE_ERR_CORRUPT);
+        if (last_cta) {
+          seg_done[seg] = 0;
+          __threadfence();   // the other CTAs' partials (published before their count) are read next
+        } else if (done > (unsigned)(c1 - c0)) {
+          raise_status(dev_status, VARRATE_ERR_CORRUPT);
+        }
       }
       __syncthreads();
       if (last_cta) {
-        __threadfence();
         if (!combine_segment(*reinterpret_cast<CombSmem*>(ring), &bar_comb, n_comb & 1u, part, c0, c1, seg,
                              qin + ((long long)b * s.H + (long long)g * s.grp) * kHeadDim,
                              basis_v + ((long long)layer * s.G + g) * kHeadDim * kHeadDim,
