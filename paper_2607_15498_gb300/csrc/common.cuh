@@ -57,11 +57,11 @@ __device__ __forceinline__ void load8_stream(const float* p, float (&f)[8]) {
 
 __device__ __forceinline__ int64_t pad8(int64_t n) { return (n + 7) & ~int64_t(7); }
 
-// Read-only 32-bit global load issued exactly where it is written (volatile: the compiler may not
+// Read-only 16-byte global load issued exactly where it is written (volatile: the compiler may not
 // sink it past later barriers), so its latency overlaps with the work that follows.
-__device__ __forceinline__ uint32_t ld_nc_early(const uint32_t* p) {
-  uint32_t v;
-  asm volatile("ld.global.nc.u32 %0, [%1];\n" : "=r"(v) : "l"(p));
+__device__ __forceinline__ uint4 ld_nc_early_v4(const uint4* p) {
+  uint4 v;
+  asm volatile("ld.global.nc.v4.u32 {%0,%1,%2,%3}, [%4];\n" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "l"(p));
   return v;
 }
 

@@ -179,32 +179,38 @@ struct RotRegs {
   uint32_t bq[kHeadDim / 16][2];   // q (B fragments; zero for padded heads)
 };
 
+// The MMA sums over k, so any one-to-one assignment of U_K's columns to the k slots of the
+// fragments gives the same product as long as q uses the same assignment. Lane (g8, c) holds the
+// 32 columns {32 i + 8 c + t : i < 4, t < 8} of its rows: four 16-byte loads per row, and the four
+// lanes of a row read 64 contiguous bytes. Column 32 i + 8 c + t feeds k-step kc = 2 i + t / 4, as
+// fragment register a0 (t % 4 < 2) or a2 (t % 4 >= 2).
 __device__ __forceinline__ void rot_load(RotRegs& rr, const __nv_bfloat16* __restrict__ U,
                                          const __nv_bfloat16* __restrict__ q, int grp, int warp, int lane) {
   const int g8 = lane >> 2, c = lane & 3, j0 = warp * 16;
-  const uint32_t* Uw = reinterpret_cast<const uint32_t*>(U);
-  const uint32_t* qw = reinterpret_cast<const uint32_t*>(q + (long long)(g8 < grp ? g8 : 0) * kHeadDim);
+  const uint4* u0 = reinterpret_cast<const uint4*>(U + (long long)(j0 + g8) * kHeadDim) + c;
+  const uint4* u1 = reinterpret_cast<const uint4*>(U + (long long)(j0 + g8 + 8) * kHeadDim) + c;
+  const uint4* qr = reinterpret_cast<const uint4*>(q + (long long)(g8 < grp ? g8 : 0) * kHeadDim) + c;
 #pragma unroll
-  for (int kc = 0; kc < kHeadDim / 16; ++kc) {
-    const int i0 = kc * 16;
-    rr.a[kc][0] = ld_nc_early(Uw + ((j0 + g8) * kHeadDim + i0 + 2 * c) / 2);
-    rr.a[kc][1] = ld_nc_early(Uw + ((j0 + g8 + 8) * kHeadDim + i0 + 2 * c) / 2);
-    rr.a[kc][2] = ld_nc_early(Uw + ((j0 + g8) * kHeadDim + i0 + 2 * c + 8) / 2);
-    rr.a[kc][3] = ld_nc_early(Uw + ((j0 + g8 + 8) * kHeadDim + i0 + 2 * c + 8) / 2);
-    rr.bq[kc][0] = ld_nc_early(qw + (i0 + 2 * c) / 2);
-    rr.bq[kc][1] = ld_nc_early(qw + (i0 + 2 * c + 8) / 2);
+  for (int i = 0; i < 4; ++i) {
+    const uint4 x = ld_nc_early_v4(u0 + 4 * i), y = ld_nc_early_v4(u1 + 4 * i), z = ld_nc_early_v4(qr + 4 * i);
+    rr.a[2 * i][0] = x.x; rr.a[2 * i][2] = x.y; rr.a[2 * i + 1][0] = x.z; rr.a[2 * i + 1][2] = x.w;
+    rr.a[2 * i][1] = y.x; rr.a[2 * i][3] = y.y; rr.a[2 * i + 1][1] = y.z; rr.a[2 * i + 1][3] = y.w;
+    rr.bq[2 * i][0] = z.x; rr.bq[2 * i][1] = z.y; rr.bq[2 * i + 1][0] = z.z; rr.bq[2 * i + 1][1] = z.w;
   }
 }
 
 __device__ __forceinline__ void rot_compute(SegSmem& sm, const RotRegs& rr, int grp, int warp, int lane) {
   const int g8 = lane >> 2, c = lane & 3, j0 = warp * 16;
   const float scale = kLog2e * rsqrtf((float)kHeadDim);
-  float d[4] = {0.f, 0.f, 0.f, 0.f};
+  float e[2][4] = {};   // even and odd k-steps: two independent MMA chains
 #pragma unroll
   for (int kc = 0; kc < kHeadDim / 16; ++kc) {
     const uint32_t b0 = g8 < grp ? rr.bq[kc][0] : 0u, b1 = g8 < grp ? rr.bq[kc][1] : 0u;
-    mma_bf16_16816(d, rr.a[kc], b0, b1);
+    mma_bf16_16816(e[kc & 1], rr.a[kc], b0, b1);
   }
+  float d[4];
+#pragma unroll
+  for (int t = 0; t < 4; ++t) d[t] = e[0][t] + e[1][t];
   // d: rows j0+g8 (+8), heads 2c, 2c+1
   sm.qt[2 * c][j0 + g8] = d[0] * scale;
   sm.qt[2 * c + 1][j0 + g8] = d[1] * scale;
