@@ -57,6 +57,21 @@ constexpr float kSlack = 8.f;                // headroom of the running max, log
 // bandwidth, so ranges that straddle segments are shortened by that much.
 constexpr long long kSegCost = 98304;
 
+// 64-bit integer division is slow on this GPU (it goes through the FP64 pipe), so the cost-line
+// arithmetic avoids it. n / d for d < 2^16 by long division in 16-bit digits: four 32-bit divisions.
+__device__ __forceinline__ unsigned long long udiv_small(unsigned long long n, uint32_t d) {
+  unsigned long long q = 0;
+  uint32_t r = 0;
+#pragma unroll
+  for (int sh = 48; sh >= 0; sh -= 16) {
+    const uint32_t cur = (r << 16) | (uint32_t)((n >> sh) & 0xFFFFu);   // r < d < 2^16
+    const uint32_t qd = cur / d;
+    r = cur - qd * d;
+    q = (q << 16) | qd;
+  }
+  return q;
+}
+
 struct SegSmem {
   alignas(16) uint32_t qfrag[kHeadDim / 16][32][4];   // per j-chunk, per lane: b0 hi, b1 hi, b0 lo, b1 lo (read as uint4)
   alignas(16) float qt[kHeadsPad][kHeadDim];          // rotated, scaled queries (fp32)
@@ -88,7 +103,7 @@ __device__ __forceinline__ void bucket_range(const SegSmem& sm, int r, long long
     if (x <= 0) return 0;
     const unsigned long long a = ((unsigned long long)x + ISL - 1) / ISL;
     if (a < (1ull << 31)) return (long long)(((uint32_t)a + (uint32_t)r - 1u) / (uint32_t)r);
-    return (long long)((a + r - 1) / r);
+    return (long long)udiv_small(a + r - 1, (uint32_t)r);
   };
   i0 = items_before(lo - b0);
   i1 = items_before(hi - b0);
@@ -234,23 +249,32 @@ __device__ void build_qfrag(SegSmem& sm, int tid) {
 }
 
 // Start of CTA c's range on a cost line of T elements cut into C equal ranges: floor(T c / C).
-// The launcher guarantees T * C < 2^63.
+// The launcher guarantees T * C < 2^63 and C <= kMaxCtas < 2^16.
 __device__ __forceinline__ long long cut_at(long long T, long long c, int C) {
-  return (long long)(((unsigned long long)T * (unsigned long long)c) / (unsigned long long)C);
+  return (long long)udiv_small((unsigned long long)T * (unsigned long long)c, (uint32_t)C);
 }
 
-// CTAs whose cost range [cuts[c], cuts[c + 1]) meets [P, P + W): c0..c1 (W > 0, P + W <= T).
-// With cuts[c] = floor(T c / C): cuts[c + 1] > P  <=>  c + 1 >= ceil((P + 1) C / T), and
-// cuts[c] > P + W - 1  <=>  c >= ceil((P + W) C / T); both products stay below T C < 2^62.
-__device__ __forceinline__ void seg_cta_range(long long T, int C, long long P, long long W, int& c0,
-                                              int& c1) {
-  const unsigned long long t = (unsigned long long)T, cc = (unsigned long long)C;
-  c0 = (int)(((unsigned long long)(P + 1) * cc + t - 1) / t) - 1;
-  const unsigned long long f = ((unsigned long long)(P + W) * cc + t - 1) / t;
-  c1 = (int)(f < cc ? f : cc) - 1;
+// CTAs whose cost range [cuts[c], cuts[c + 1]) meets [P, P + W): c0..c1 (W > 0, P + W <= T,
+// cuts[c] = floor(T c / C)). c0 is the first c with cuts[c + 1] > P, i.e. ceil((P + 1) C / T) - 1,
+// and c1 + 1 the first c with cuts[c] > P + W - 1, i.e. ceil((P + W) C / T) (at most C). Both are
+// estimated in fp32 and then corrected against the table, which makes them exact.
+__device__ __forceinline__ void seg_cta_range(const long long* cuts, long long T, int C, long long P,
+                                              long long W, int& c0, int& c1) {
+  int c = (int)ceilf((float)(P + 1) * (float)C / (float)T) - 1;
+  c = max(0, min(C - 1, c));
+  while (c > 0 && cuts[c] > P) --c;
+  while (c < C - 1 && cuts[c + 1] <= P) ++c;
+  c0 = c;
+  const long long X = P + W - 1;
+  c = min((int)ceilf((float)(P + W) * (float)C / (float)T), C) - 1;
+  c = max(0, min(C - 1, c));
+  while (c < C - 1 && cuts[c + 1] <= X) ++c;
+  while (c > 0 && cuts[c] > X) --c;
+  c1 = c;
 }
 
 constexpr int kMaxCtas = 1024;   // grid size bound (64-bit cost-line arithmetic)
+static_assert(kMaxCtas < (1 << 16), "udiv_small divides by the grid size");
 
 struct CombSmem {   // aliases the ring while the last CTA of a segment combines it
   alignas(128) __nv_bfloat16 us[kHeadDim * kHeadDim];   // U_V[g], row j (one bulk copy)
@@ -466,7 +490,12 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
       if (segP[mid + 1] > lo_g) hi_b = mid; else lo_b = mid + 1;
     }
     b = lo_b;
-    if (b < s.B) g = (int)((lo_g - segP[b]) / (segW[b] + kSegCost));
+    if (b < s.B) {   // g = floor(x / w), estimated in fp32 and corrected
+      const long long x = lo_g - segP[b], w = segW[b] + kSegCost;
+      g = (int)((float)x / (float)w);
+      while (g > 0 && (long long)g * w > x) --g;
+      while ((long long)(g + 1) * w <= x) ++g;
+    }
   }
   auto seg_start = [&](int bb, int gg) { return segP[bb] + gg * (segW[bb] + kSegCost) + kSegCost; };
   bool more = b < s.B && seg_start(b, g) < hi_g;
@@ -541,7 +570,7 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
         if (issue_chunk(pr, sm, cK, cV, ring_w + ((n_issued + i) % ST) * STAGE,
                         &bars[(n_issued + i) % ST], total, lane)) ++n_pending;
       int c0, c1;   // the CTAs that share this segment (their partials are merged by the last one)
-      seg_cta_range(T, C, P, W, c0, c1);
+      seg_cta_range(cuts, T, C, P, W, c0, c1);
       __syncwarp();
       rot_compute(sm, rr, s.grp, warp, lane);
       __syncthreads();
