@@ -141,7 +141,8 @@ struct Prod {
 // Returns false (and issues nothing) when the stream is exhausted.
 __device__ __forceinline__ bool issue_chunk(Prod& p, const SegSmem& sm, const __nv_bfloat16* cK,
                                             const __nv_bfloat16* cV, uint32_t stage_addr,
-                                            uint64_t* bar, int total, int lane) {
+                                            uint64_t* bar, int total, int lane, uint64_t policy,
+                                            bool fence = true) {
   if (p.k >= total) return false;
   const int r = p.item.r;
   const long long n8 = pad8(sm.cnt[r]);
@@ -153,9 +154,9 @@ __device__ __forceinline__ bool issue_chunk(Prod& p, const SegSmem& sm, const __
   if (lane == 0) {
     const uint32_t bytes = (uint32_t)(rows * tl * 2);           // rows j0.. of the tile: contiguous
     mbar_arrive_expect_tx(bar, bytes);
-    fence_proxy_async_smem();  // the generic reads above precede the async write
+    if (fence) fence_proxy_async_smem();  // the generic reads above precede the async write
     bulk_g2s_hint(stage_addr, (p.phase ? cV : cK) + sm.base[r] + t0 * r + (long long)j0 * tl, bytes, bar,
-                  l2_evict_first_policy());
+                  policy);
   }
   __syncwarp();   // lane 0 branched off: reconverge before the next warp-wide instruction
   const int nj = (r + CH - 1) / CH;
@@ -432,6 +433,7 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int g8 = lane >> 2, c = lane & 3;
   const int C = gridDim.x, cta = blockIdx.x;
+  const uint64_t policy = l2_evict_first_policy();   // coefficient chunks are read once
 
   // the next grid in the stream may be scheduled now: it only starts on SMs this grid has left,
   // and waits (griddepcontrol.wait) for this grid to finish before it reads anything
@@ -567,8 +569,9 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
       Item cons = pr.item;
 #pragma unroll
       for (int i = 0; i < ST - 1; ++i)
+        // the ring was zeroed and fenced before the segment began: no fence for these
         if (issue_chunk(pr, sm, cK, cV, ring_w + ((n_issued + i) % ST) * STAGE,
-                        &bars[(n_issued + i) % ST], total, lane)) ++n_pending;
+                        &bars[(n_issued + i) % ST], total, lane, policy, false)) ++n_pending;
       int c0, c1;   // the CTAs that share this segment (their partials are merged by the last one)
       seg_cta_range(cuts, T, C, P, W, c0, c1);
       __syncwarp();
@@ -589,7 +592,7 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
         ++n_issued;
         --n_pending;
         if (issue_chunk(pr, sm, cK, cV, ring_w + ((n_issued + ST - 2) % ST) * STAGE,
-                        &bars[(n_issued + ST - 2) % ST], total, lane)) ++n_pending;
+                        &bars[(n_issued + ST - 2) % ST], total, lane, policy)) ++n_pending;
       };
 
       while (cons_k < total && !timed_out) {
