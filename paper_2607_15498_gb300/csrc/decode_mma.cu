@@ -45,7 +45,7 @@ constexpr int kMaxR = kHeadDim;
 constexpr int NW = 8;                 // warps per CTA
 constexpr int ST = 3;                 // ring stages per warp
 constexpr int ISL = 128;              // slots per item
-constexpr int CH = 32;                // coefficient rows per chunk
+constexpr int CH = 32;                // coefficient rows per chunk of a full 128-slot tile
 constexpr int STAGE = CH * ISL * 2;   // one chunk: up to 32 rows of a 128-slot tile
 constexpr int kPartStride = kHeadDim + 4;   // o~[128], max, sum, pad: rows 16-byte aligned
 constexpr int kHeadsPad = 8;
@@ -128,6 +128,13 @@ __device__ __forceinline__ Item item_at(const SegSmem& sm, int k) {
   return x;
 }
 
+// Rows per chunk of a tile of tl slots, as log2: as many rows as fill one 8 KB stage (32 rows of a
+// full 128-slot tile, 64 of a tile of at most 64 slots, all 128 of a tile of at most 32). The
+// sparse high-rank buckets end in short tiles; reading them in few chunks keeps their items from
+// being a chain of small, latency-bound copies.
+__device__ __forceinline__ int chunk_lg(int tl) { return tl > 64 ? 5 : (tl > 32 ? 6 : 7); }
+static_assert((ISL * 2) << 5 == STAGE, "a full tile's chunk fills a stage");
+
 // Producer cursor: which chunk of which item comes next in this warp's stream.
 struct Prod {
   int k;       // item index (CTA-local)
@@ -136,7 +143,7 @@ struct Prod {
   int jc;      // 16-row chunk index
 };
 
-// Issue the next chunk of this warp's stream into `stage`: rows j0..j0+31 of one 128-slot tile are
+// Issue the next chunk of this warp's stream into `stage`: consecutive rows of one tile are
 // contiguous in the packed layout, so one bulk copy moves the whole chunk.
 // Returns false (and issues nothing) when the stream is exhausted.
 __device__ __forceinline__ bool issue_chunk(Prod& p, const SegSmem& sm, const __nv_bfloat16* cK,
@@ -148,8 +155,9 @@ __device__ __forceinline__ bool issue_chunk(Prod& p, const SegSmem& sm, const __
   const long long n8 = pad8(sm.cnt[r]);
   const long long t0 = (long long)p.item.it * ISL;            // first slot of the tile
   const long long tl = min((long long)ISL, n8 - t0);            // slots in the tile (multiple of 8)
-  const int j0 = p.jc * CH;
-  const int rows = min(CH, r - j0);
+  const int lgc = chunk_lg((int)tl);
+  const int j0 = p.jc << lgc;
+  const int rows = min(1 << lgc, r - j0);
   // callers have __syncwarp()ed: every lane's ldmatrix reads of this stage are done
   if (lane == 0) {
     const uint32_t bytes = (uint32_t)(rows * tl * 2);           // rows j0.. of the tile: contiguous
@@ -159,7 +167,7 @@ __device__ __forceinline__ bool issue_chunk(Prod& p, const SegSmem& sm, const __
                   policy);
   }
   __syncwarp();   // lane 0 branched off: reconverge before the next warp-wide instruction
-  const int nj = (r + CH - 1) / CH;
+  const int nj = (r + (1 << lgc) - 1) >> lgc;
   if (++p.jc == nj) {
     p.jc = 0;
     if (++p.phase == 2) {
@@ -597,7 +605,6 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
 
       while (cons_k < total && !timed_out) {
         const int r = cons.r;
-        const int nj = (r + CH - 1) / CH;
         const long long n_real = sm.cnt[r] - (long long)cons.it * ISL;   // real slots of this item
         // tile geometry (packed layout, coef_offset): rows of tl slots, 8-slot group g of row j
         // stored at position (g + j) mod (tl / 8)
@@ -605,6 +612,8 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
         const int ng = tl >> 3;
         const bool full_tile = ng == 16;
         const uint32_t row_bytes = (uint32_t)tl * 2u;
+        const int lgc = chunk_lg(tl);                   // same chunking as the producer
+        const int nj = (r + (1 << lgc) - 1) >> lgc;
         float sc[ISL / 16][4];
 #pragma unroll
         for (int t = 0; t < ISL / 16; ++t) sc[t][0] = sc[t][1] = sc[t][2] = sc[t][3] = 0.f;
@@ -614,10 +623,9 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
           if (!wait_chunk()) break;
           const uint32_t st_addr = ring_w + (n_issued % ST) * STAGE;
           const int m = lane >> 3, r8 = lane & 7;
-#pragma unroll
-          for (int ks = 0; ks < CH / 16; ++ks) {
-            const int j16 = jc * CH + ks * 16;
-            if (j16 >= r) break;                        // warp-uniform
+          const int j0 = jc << lgc, j1 = min(r, j0 + (1 << lgc));
+#pragma unroll 2
+          for (int j16 = j0; j16 < j1; j16 += 16) {
             uint4 qf = *reinterpret_cast<const uint4*>(&sm.qfrag[j16 >> 4][lane][0]);
             if (j16 + 16 > r) {                          // warp-uniform: rows >= r in this k-step
               const int jb = j16 + 2 * c;
@@ -625,8 +633,8 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
               qf.y = keep_rows(qf.y, jb + 8, r); qf.w = keep_rows(qf.w, jb + 8, r);
             }
             // this lane's row of the 8x8 matrices: coefficient j, staged at row (j - chunk start)
-            const int jrow = ks * 16 + (m >> 1) * 8 + r8;
-            const int j = jc * CH + jrow;
+            const int jrow = (j16 - j0) + (m >> 1) * 8 + r8;
+            const int j = j0 + jrow;
             const uint32_t row_addr = st_addr + jrow * row_bytes;
             uint32_t a[ISL / 16][4];
             int pg = full_tile ? (((m & 1) + j) & 15) : (((m & 1) + j) % ng);   // slot group 2 mt + (m & 1)
@@ -695,18 +703,25 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
         Ls[1] = Ls[1] * corr[1] + lsum[1];
 
         // ---- V chunks: weighted coefficient rows (rows >= r masked in the A fragment)
-#pragma unroll
-        for (int jc = 0; jc < kHeadDim / CH; ++jc) {
-          if (jc >= nj) break;
-          if (!wait_chunk()) break;
-          const uint32_t st_addr = ring_w + (n_issued % ST) * STAGE;
+        {
+          int left = 0;             // rows of the current chunk not used yet
+          int j0 = 0;               // first row of the current chunk
+          uint32_t st_addr = 0;
+          bool ok = true;
           const int m = lane >> 3, r8 = lane & 7;
 #pragma unroll
-          for (int ks = 0; ks < CH / 16; ++ks) {
-            const int jt = jc * (CH / 16) + ks;         // 16-row tile of o~
-            if (jt * 16 >= r) break;                    // warp-uniform
-            const int jrow = ks * 16 + (m & 1) * 8 + r8;
-            const int j = jc * CH + jrow;
+          for (int jt = 0; jt < kHeadDim / 16; ++jt) {   // 16-row tile of o~
+            if (jt * 16 >= r) break;                     // warp-uniform
+            if (left == 0) {                             // the tile starts a chunk
+              if (jt > 0) { __syncwarp(); next_chunk(); }
+              if (!wait_chunk()) { ok = false; break; }
+              st_addr = ring_w + (n_issued % ST) * STAGE;
+              j0 = jt * 16;
+              left = 1 << lgc;
+            }
+            left -= 16;
+            const int jrow = (jt * 16 - j0) + (m & 1) * 8 + r8;
+            const int j = j0 + jrow;
             const uint32_t row_addr = st_addr + jrow * row_bytes;
             const bool keep0 = jt * 16 + g8 < r, keep1 = jt * 16 + g8 + 8 < r;
             float t1[4] = {0.f, 0.f, 0.f, 0.f};
@@ -728,8 +743,7 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
 #pragma unroll
             for (int e = 0; e < 4; ++e) oacc[jt][e] += t1[e];
           }
-          __syncwarp();
-          next_chunk();
+          if (ok) { __syncwarp(); next_chunk(); }         // the last chunk of the item
         }
         cons_k += NW;
         if (cons_k < total) cons = item_at(sm, cons_k);
