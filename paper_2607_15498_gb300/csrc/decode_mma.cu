@@ -55,7 +55,7 @@ constexpr float kSlack = 8.f;                // headroom of the running max, log
 // segment pays its set-up (tables, query rotation, pipeline ramp, partial write, and for one CTA
 // the combine), about as long as streaming this many coefficients at a CTA's share of HBM
 // bandwidth, so ranges that straddle segments are shortened by that much.
-constexpr long long kSegCost = 98304;
+constexpr long long kSegCost = 90112;
 
 // 64-bit integer division is slow on this GPU (it goes through the FP64 pipe), so the cost-line
 // arithmetic avoids it. n / d for d < 2^16 by long division in 16-bit digits: four 32-bit divisions.
