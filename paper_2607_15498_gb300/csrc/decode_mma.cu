@@ -9,8 +9,8 @@
 // ranges, so every SM moves the same number of bytes. A CTA walks the (sequence, head) segments its
 // range touches; per segment it rotates the query with mma.sync (U_K tile x q), then its warps take
 // 128-slot items (one tile of the packed layout) of one rank bucket round-robin. An item of rank r
-// is 2 * ceil(r/32) chunks of up to 32 coefficient rows x 128 slots (8 KB), each one contiguous
-// block: all K chunks, then all V chunks.
+// is read as K chunks then V chunks of up to 8 KB each (32 rows of a full tile, 64 or 128 rows of a
+// short one), each one contiguous block.
 //
 // Memory path. Each warp owns a 3-stage shared-memory ring filled by one 1-D TMA bulk copy per
 // chunk that completes on a per-stage mbarrier; the warp stays 2 chunks ahead of the chunk it
@@ -57,8 +57,9 @@ constexpr float kSlack = 8.f;                // headroom of the running max, log
 // bandwidth, so ranges that straddle segments are shortened by that much.
 constexpr long long kSegCost = 90112;
 
-// 64-bit integer division is slow on this GPU (it goes through the FP64 pipe), so the cost-line
-// arithmetic avoids it. n / d for d < 2^16 by long division in 16-bit digits: four 32-bit divisions.
+// A 64-bit integer division is a long instruction sequence (measured ~600 cycles here), so the
+// cost-line arithmetic avoids it. n / d for d < 2^16 by long division in 16-bit digits: four
+// 32-bit divisions.
 __device__ __forceinline__ unsigned long long udiv_small(unsigned long long n, uint32_t d) {
   unsigned long long q = 0;
   uint32_t r = 0;
