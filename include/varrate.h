@@ -183,7 +183,12 @@ varrate_status varrate_encode(const varrate_config* cfg, const void* q_win, cons
  *           call writes before it reads. So one workspace serves any number of later decode calls
  *           (any shape), provided they are ordered on one stream. A call that finds a counter
  *           that is not zero raises VARRATE_ERR_CORRUPT in *dev_status: zero the workspace again
- *           before its next use. */
+ *           before its next use.
+ * In bf16 the call's kernel is launched with programmatic stream serialization and allows the next
+ * kernel on `stream` to be scheduled while it runs: a following kernel launched with that attribute
+ * must wait for it (griddepcontrol.wait / cudaGridDependencySynchronize) before it reads `out` or
+ * `*dev_status`. Kernels launched without the attribute, and every other stream operation, still
+ * start only after it has finished. */
 varrate_status varrate_decode_attn(const varrate_config* cfg, const varrate_packed* cache,
                                    const void* basis_k, const void* basis_v, const void* q,
                                    int32_t layer, const void* tail_k, const void* tail_v,
