@@ -65,8 +65,8 @@ def salience_raw(q_win: np.ndarray, k: np.ndarray, group: int) -> np.ndarray:
 
     q_win: [w][H][d] queries of the last w tokens (window query q sits at position N - w + q).
     k:     [G][N][d] keys; query head h reads KV head h // group.
-    For every window query and head, alpha = softmax over t <= p of <q, k_t> / sqrt(d) (the
-    tokens seen so far, Sec. 3.1 "Attention and the KV cache"); s_t is the mean of alpha over the
+    For every window query and head, alpha = softmax over t <= p of <q, k_t> / sqrt(d) (every
+    token up to the query's own position, Sec. 3.1 "Attention and the KV cache"); s_t is the mean of alpha over the
     w queries and H heads. Returns s for the coded set t in [0, N - w), fp64."""
     q_win = np.asarray(q_win, dtype=np.float64)
     k = np.asarray(k, dtype=np.float64)
