@@ -5,6 +5,22 @@ Functions keep the C names and argument order; tensor arguments are torch tensor
 owned by the caller) or ``None`` for NULL, and ``stream`` defaults to torch's current stream.
 Importing this module does not load the library; the first call does, and it raises if the
 library has not been built (there is no CPU fallback).
+
+Typical use (one encode of a prompt's cache, then one decode call per layer and step)::
+
+    cfg = make_config(n_layers, n_kv_heads, group, n_ctx, batch=B, budget_frac=0.2, r_min=16,
+                      window=32, dtype=BF16)
+    packed = PackedCache.allocate(cfg, "cuda")            # static upper bound: no host sync later
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    check(varrate_encode(cfg, q_win, k, v, basis_k, basis_v, None, packed, None, status,
+                         workspace(cfg, CALL_ENCODE)), "varrate_encode")
+    ws = workspace(cfg, CALL_DECODE)                      # zero-filled; reusable by every decode call
+    check(varrate_decode_attn(cfg, packed, basis_k, basis_v, q, layer, None, None, 0, out, status,
+                              ws), "varrate_decode_attn")
+    # after a synchronise: status.item() is OK (0), FLOOR_BINDS (1) or a negative error
+
+Shapes: q_win [B][L][w][H][d], k and v [B][L][G][N][d], bases [L][G][d][d] (row j = basis vector
+j), q and out [B][H][d]; every tensor contiguous on the GPU and 16-byte aligned.
 """
 from __future__ import annotations
 
