@@ -361,6 +361,27 @@ def decode_recon(q, coef_k, coef_v, ranks, basis_k, basis_v, tail_k=None, tail_v
     return attention(q, kh, vh)
 
 
+def decode_window(q, coef_k, coef_v, ranks, basis_k, basis_v, tail_k, tail_v):
+    """Decode attention for a window of n_q consecutive new tokens in one call (the multi-query
+    form of the exact-tail decode: the recent tokens are kept exact, Sec. 3.1 "Residual codec").
+
+    q [n_q][H][d] are the queries of the last n_q tokens of the exact tail tail_k, tail_v
+    [G][n_tail][d] (n_tail >= n_q). Query i sits at tail position n_tail - n_q + i and, as in
+    causal attention (Sec. 3.1 "Attention and the KV cache"), attends to every cached token and to
+    the tail tokens up to and including its own position. Returns [n_q][H][d]."""
+    q = np.asarray(q, dtype=np.float64)
+    n_q = q.shape[0]
+    n_tail = np.asarray(tail_k).shape[1]
+    if n_q > n_tail:
+        raise ValueError("every window query is one of the tail tokens")
+    out = np.zeros(q.shape)
+    for i in range(n_q):
+        m = n_tail - n_q + i + 1                    # tail tokens visible to query i
+        out[i] = decode_coef(q[i], coef_k, coef_v, ranks, basis_k, basis_v,
+                             np.asarray(tail_k)[:, :m], np.asarray(tail_v)[:, :m])
+    return out
+
+
 # --------------------------------------------------------------------------- whole layer
 
 def encode_layer(q_win, k, v, basis_k, basis_v, group, budget_frac, r_min, pool_len=5,

@@ -336,6 +336,60 @@ def test_decode_with_exact_tail():
     np.testing.assert_allclose(full, want, atol=1e-10)
 
 
+def _sdpa_window(q, k, v, n_tail):
+    """Causal attention of the last n_q of n = N + n_tail tokens, from torch SDPA (fp64):
+    query i (token n - n_q + i) sees tokens 0 .. n - n_q + i. q [n_q][H][d]; k, v [G][n][d]."""
+    n_q, H, d = q.shape
+    G, n, _ = k.shape
+    kk = torch.as_tensor(k).repeat_interleave(H // G, dim=0)[None]      # [1][H][n][d]
+    vv = torch.as_tensor(v).repeat_interleave(H // G, dim=0)[None]
+    qq = torch.as_tensor(q).permute(1, 0, 2)[None]                      # [1][H][n_q][d]
+    mask = torch.arange(n)[None, :] <= (n - n_q + torch.arange(n_q))[:, None]
+    out = torch.nn.functional.scaled_dot_product_attention(qq, kk, vv, attn_mask=mask[None, None])
+    return out[0].permute(1, 0, 2).numpy()
+
+
+def _window_case(n_ctx=160, n_tail=9, n_q=4, seed=21):
+    wl = synth.workload("tiny", n_ctx=n_ctx, window=8, n_kv_heads=2)
+    k, v = synth.layer_kv(wl, 0, 0, out_dtype=torch.float64)
+    k, v = k.numpy(), v.numpy()
+    uk, uv = synth.bases(wl, 0)
+    rng = np.random.default_rng(seed)
+    q = rng.standard_normal((n_q, wl.n_q_heads, wl.head_dim))
+    tk = rng.standard_normal((2, n_tail, wl.head_dim))
+    tv = rng.standard_normal((2, n_tail, wl.head_dim))
+    ck = np.stack([O.project(k[g], uk[g]) for g in range(2)])
+    cv = np.stack([O.project(v[g], uv[g]) for g in range(2)])
+    return k, v, uk, uv, q, tk, tv, ck, cv, rng
+
+
+def test_window_decode_full_rank_is_causal_attention():
+    """At full rank the window decode is causal attention over cache + tail (torch SDPA, masked)."""
+    k, v, uk, uv, q, tk, tv, ck, cv, _ = _window_case()
+    got = O.decode_window(q, ck, cv, np.full(k.shape[1], 128), uk, uv, tk, tv)
+    want = _sdpa_window(q, np.concatenate([k, tk], 1), np.concatenate([v, tv], 1), tk.shape[1])
+    np.testing.assert_allclose(got, want, atol=1e-10)
+
+
+def test_window_decode_sees_no_later_token():
+    """Query i is unchanged when the tail tokens after its own position change, and changes when
+    an earlier one does; with n_q = 1 it is the single-query decode over the whole tail."""
+    k, v, uk, uv, q, tk, tv, ck, cv, rng = _window_case()
+    ranks = rng.integers(16, 129, size=k.shape[1])
+    n_tail, n_q = tk.shape[1], q.shape[0]
+    base = O.decode_window(q, ck, cv, ranks, uk, uv, tk, tv)
+    tk2, tv2 = tk.copy(), tv.copy()
+    tk2[:, -1] += 3.0
+    tv2[:, -1] -= 2.0                                   # the last query's own token
+    moved = O.decode_window(q, ck, cv, ranks, uk, uv, tk2, tv2)
+    np.testing.assert_array_equal(moved[:-1], base[:-1])
+    assert np.abs(moved[-1] - base[-1]).max() > 1e-6
+    one = O.decode_window(q[-1:], ck, cv, ranks, uk, uv, tk, tv)
+    np.testing.assert_allclose(one[0], O.decode_coef(q[-1], ck, cv, ranks, uk, uv, tk, tv), atol=1e-12)
+    with pytest.raises(ValueError):
+        O.decode_window(np.zeros((n_tail + 1,) + q.shape[1:]), ck, cv, ranks, uk, uv, tk, tv)
+
+
 def test_decode_single_token_and_flat_scores():
     d = 16
     rng = np.random.default_rng(8)
