@@ -167,3 +167,19 @@ def test_binding_fails_loudly_without_library(tmp_path, monkeypatch):
     monkeypatch.setattr(V, "LIB_PATH", str(tmp_path / "missing.so"))
     with pytest.raises(RuntimeError, match="no CPU fallback"):
         V.lib()
+
+
+def test_packed_cache_and_workspace_helpers(vlib):
+    """The binding's allocators give the documented shapes, 16-byte aligned buffers and a
+    zero-filled workspace (allocated here on the host: only the layout is checked)."""
+    cfg = vlib.make_config(2, 3, 4, 1000, batch=2, dtype=vlib.BF16)
+    p = vlib.PackedCache.allocate(cfg, "cpu")
+    cap = vlib.varrate_packed_cap_elems(cfg)
+    assert p.cap_elems == cap and cap % 8 == 0
+    assert tuple(p.coef.shape) == (2, 2, 3, 2, cap) and p.coef.dtype == vlib.torch.bfloat16
+    assert tuple(p.bucket_count.shape) == (2, 2, 129) and tuple(p.bucket_base.shape) == (2, 2, 130)
+    for t in (p.coef, p.bucket_count, p.bucket_base, p.perm, p.pos, p.ranks):
+        assert t.data_ptr() % 16 == 0
+    ws = vlib.workspace(cfg, vlib.CALL_DECODE, "cpu")
+    assert ws.numel() >= vlib.varrate_workspace_bytes(cfg, vlib.CALL_DECODE)
+    assert int(vlib.torch.count_nonzero(ws)) == 0
