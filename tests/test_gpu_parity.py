@@ -219,6 +219,11 @@ def test_decode_with_exact_tail(inputs):
     _decode_check(CASES["llama_ragged"], inputs["llama_ragged"], n_tail=37, n_steps=2)
 
 
+def test_decode_with_long_exact_tail(inputs):
+    # more than 64 tail tokens: the bf16 call takes the general split-and-combine kernels
+    _decode_check(CASES["llama_ragged"], inputs["llama_ragged"], n_tail=100, n_steps=1)
+
+
 def test_decode_uniform_mode(inputs):
     _decode_check(CASES["llama_ragged"], inputs["llama_ragged"], mode=O.UNIFORM, n_steps=2)
 
