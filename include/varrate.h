@@ -11,7 +11,11 @@
  *  - Every tensor argument is a caller-owned DEVICE pointer (CUDA global memory), row-major and
  *    densely packed in the layout stated next to it, and 16-byte aligned (as cudaMalloc and
  *    PyTorch allocations are); a misaligned pointer is VARRATE_ERR_ARG. The library never
- *    allocates or frees device memory and keeps no state between calls (reentrant).
+ *    allocates or frees device memory. Calls are reentrant and thread-safe. Across calls the
+ *    library keeps only per-process values that do not change results: each device's SM count,
+ *    the driver entry point that encodes TMA descriptors, a counter that tags every decode call
+ *    (see varrate_decode_attn), and the device address of the allocation-free entry point's
+ *    scratch array. All are held in atomics.
  *  - `stream` is a cudaStream_t passed as void* (NULL = the legacy default stream). Every call
  *    only enqueues work on `stream` and returns without synchronising.
  *  - The return value reports what the host can see: bad arguments (VARRATE_ERR_ARG), a workspace
@@ -51,7 +55,8 @@ typedef enum {
   VARRATE_ERR_CUDA = -3,         /* a CUDA launch or runtime call failed */
   VARRATE_ERR_TIMEOUT = -4,      /* a bounded device-side wait gave up */
   VARRATE_ERR_UNSUPPORTED = -5,  /* a shape outside the limits above */
-  VARRATE_ERR_CORRUPT = -6       /* rank or layout table outside its valid range */
+  VARRATE_ERR_CORRUPT = -6       /* rank or layout table outside its valid range, or decode
+                                    completion words left inconsistent by an earlier call */
 } varrate_status;
 
 typedef enum { VARRATE_F32 = 0, VARRATE_BF16 = 1 } varrate_dtype;
@@ -175,20 +180,29 @@ varrate_status varrate_encode(const varrate_config* cfg, const void* q_win, cons
  *   (and the n_tail exact tail tokens);  o = U_V^T sum_t alpha_t c^V_t[:r_t] + sum_tail alpha v.
  *   q       [B][H][d]  one query per head per sequence
  *   tail_k/_v [B][G][n_tail][d] uncompressed tokens appended after the cache (may be NULL if
- *           n_tail == 0)
+ *           n_tail == 0); 0 <= n_tail <= 4096 (more is VARRATE_ERR_UNSUPPORTED)
  *   out     [B][H][d]  dtype
  *   ws      at least varrate_workspace_bytes(cfg, VARRATE_CALL_DECODE) bytes, zero-filled before
- *           the first decode call that uses it. Its first 16 KiB hold per-(sequence, KV head)
- *           completion counters that every call leaves at zero again; the rest is scratch that a
- *           call writes before it reads. So one workspace serves any number of later decode calls
- *           (any shape), provided they are ordered on one stream. A call that finds a counter
- *           that is not zero raises VARRATE_ERR_CORRUPT in *dev_status: zero the workspace again
- *           before its next use.
- * In bf16 the call's kernel is launched with programmatic stream serialization and allows the next
- * kernel on `stream` to be scheduled while it runs: a following kernel launched with that attribute
- * must wait for it (griddepcontrol.wait / cudaGridDependencySynchronize) before it reads `out` or
+ *           the first decode call that uses it. Its first 32 KiB hold one 64-bit completion word
+ *           per (sequence, KV head) (at most 4096): the tag of the last call that used it, the
+ *           number of thread blocks that call split the pair over, and how many have finished.
+ *           Every call leaves its words finished; the rest of the workspace is scratch that a call
+ *           writes before it reads. So one workspace serves any number of later decode calls (any
+ *           shape), provided they are ordered on one stream. Calls that overlap on one workspace
+ *           (different streams, host threads) race and give wrong results. A call that finds a
+ *           word that is neither zero nor finished (an overlapping call, a call that gave up with
+ *           VARRATE_ERR_TIMEOUT, or garbage) raises VARRATE_ERR_CORRUPT in *dev_status and re-arms
+ *           the word for itself, so the next call on the workspace is clean again without any
+ *           action by the caller; results written while the words were inconsistent are not to be
+ *           trusted. Replaying a captured launch of this call is fine: the replay keeps its tag and
+ *           finds its own finished words.
+ * Kernels: in bf16 with n_tail <= 64, batch <= 64 and batch * n_kv_heads <= 4096 one fused kernel
+ * runs. It is launched with programmatic stream serialization and allows the next kernel on
+ * `stream` to be scheduled while it runs: a following kernel launched with that attribute must wait
+ * for it (griddepcontrol.wait / cudaGridDependencySynchronize) before it reads `out` or
  * `*dev_status`. Kernels launched without the attribute, and every other stream operation, still
- * start only after it has finished. */
+ * start only after it has finished. Other shapes (and fp32) run three ordinary kernels (query
+ * rotation, split over tokens, combine), launched without that attribute. */
 varrate_status varrate_decode_attn(const varrate_config* cfg, const varrate_packed* cache,
                                    const void* basis_k, const void* basis_v, const void* q,
                                    int32_t layer, const void* tail_k, const void* tail_v,
@@ -204,11 +218,15 @@ varrate_status varrate_decode_attn(const varrate_config* cfg, const varrate_pack
  *  - Returns VARRATE_ERR_WORKSPACE when the shape needs more than 4 MiB of decode scratch
  *    (varrate_workspace_bytes(cfg, VARRATE_CALL_DECODE) > 4 MiB).
  *  - The first call on a device looks up the array's device address (once per device, for the
- *    current device); make that first call before any stream capture.
+ *    current device) and caches it; make that first call before any stream capture. After
+ *    cudaDeviceReset of a device the cached address is stale: do not call this entry point on
+ *    that device again in the process.
  *  - All calls share the one array: calls that overlap on the GPU (other streams, other host
- *    threads) race on it and must be serialised by the caller. The array starts zero-filled; its
- *    completion counters are left at zero by every call and the rest is written before it is
- *    read, so no contents carry over that matter. */
+ *    threads) race on it and must be serialised by the caller. The array starts zero-filled and
+ *    keeps the last call's contents: its completion words work as described for
+ *    varrate_decode_attn (left finished by every call; after an overlap or a timed-out call the
+ *    next call reports VARRATE_ERR_CORRUPT once and re-arms them, since the caller cannot clear
+ *    this array), and the rest is written before it is read. */
 varrate_status varrate_decode_attn_noalloc(const varrate_config* cfg, const varrate_packed* cache,
                                            const void* basis_k, const void* basis_v, const void* q,
                                            int32_t layer, const void* tail_k, const void* tail_v,

@@ -1,5 +1,6 @@
 // C ABI of the VarRate hot path (declared in include/varrate.h): argument validation, workspace
 // carving and kernel launches. No device memory is allocated here.
+#include <atomic>
 #include <initializer_list>
 #include <math.h>
 #include <stdint.h>
@@ -58,16 +59,26 @@ Shape make_shape(const varrate_config* c, int64_t cap) {
   return s;
 }
 
+// SM count of each device, cached per process (a property of the device: every thread that fills
+// an entry writes the same value).
 int num_sms() {
-  static int cached[64] = {0};
+  static std::atomic<int> cached[64];
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 148;
-  if (cached[dev] == 0) {
-    int n = 0;
+  int n = cached[dev].load(std::memory_order_relaxed);
+  if (n == 0) {
     if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 148;
-    cached[dev] = n;
+    cached[dev].store(n, std::memory_order_relaxed);
   }
-  return cached[dev];
+  return n;
+}
+
+// Tag of one decode call in the workspace's completion words: a process-wide counter, never 0.
+uint32_t next_decode_epoch() {
+  static std::atomic<uint32_t> counter{0};
+  uint32_t e = counter.fetch_add(1, std::memory_order_relaxed) + 1;
+  if (e == 0) e = counter.fetch_add(1, std::memory_order_relaxed) + 1;
+  return e;
 }
 
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
@@ -119,7 +130,7 @@ const char* varrate_status_string(int32_t st) {
     case VARRATE_ERR_CUDA: return "CUDA launch or runtime error";
     case VARRATE_ERR_TIMEOUT: return "bounded device wait timed out";
     case VARRATE_ERR_UNSUPPORTED: return "unsupported shape";
-    case VARRATE_ERR_CORRUPT: return "rank or layout table out of range";
+    case VARRATE_ERR_CORRUPT: return "rank or layout table out of range, or decode workspace left inconsistent";
     default: return "unknown status";
   }
 }
@@ -226,7 +237,7 @@ varrate_status varrate_decode_attn(const varrate_config* cfg, const varrate_pack
   if (ws_bytes_ < need || ws == nullptr) return VARRATE_ERR_WORKSPACE;
   const Shape s = make_shape(cfg, cache->cap_elems);
   vr::launch_decode(s, *cache, basis_k, basis_v, q, layer, tail_k, tail_v, n_tail, out, dev_status,
-                    ws, num_sms(), (cudaStream_t)stream);
+                    ws, next_decode_epoch(), num_sms(), (cudaStream_t)stream);
   return launched();
 }
 

@@ -25,9 +25,9 @@
 //   values   O~^T[j][head] += V[j][slot] * P^T[slot][head]      (P in bf16, <= 2^-9 relative per
 //            weight, transposed from the score fragments with movmatrix)
 // Partials (max, sum, o~[128]) per (segment, CTA) go to the workspace. The last CTA to finish a
-// segment (a per-segment counter in the workspace, which that CTA sets back to zero for the next
-// call) merges its partials, adds the exact tail, rotates back with U_V^T (staged in the idle ring)
-// and normalises, so one launch does the whole step.
+// segment (counted in a per-segment completion word in the workspace, tagged with the call's epoch)
+// merges its partials, adds the exact tail, rotates back with U_V^T (staged in the idle ring) and
+// normalises, so one launch does the whole step.
 //
 // Warps reconverge explicitly (__syncwarp) after lane-dependent code and before warp-wide
 // shuffles, votes and tensor-core fragments: left to itself a diverged warp reaching those
@@ -286,6 +286,46 @@ __device__ __forceinline__ void seg_cta_range(const long long* cuts, long long T
 constexpr int kMaxCtas = 1024;   // grid size bound (64-bit cost-line arithmetic)
 static_assert(kMaxCtas < (1 << 16), "udiv_small divides by the grid size");
 
+// Completion word of one (sequence, KV head) segment: bits 63..32 hold the epoch of the call that
+// arrived last, bits 31..16 the number of CTAs that call expects on the segment, bits 15..0 how many
+// have arrived. A word is clean when it is zero (never used) or holds a finished count. The first
+// CTA of a call replaces a clean word by (epoch, n, 1), the others count up, and the one that
+// completes the count merges the segment. Any other word (another epoch still counting, a count or
+// an expected value out of range) means an earlier call never finished or two calls overlap on
+// this workspace: the arrival raises VARRATE_ERR_CORRUPT and re-arms the word for its own call, so
+// the next call finds it clean. A replay of a captured launch keeps its epoch and finds its own
+// finished word, which is clean. Returns true for the CTA that completes the count.
+// The CTA that completes the count (it merges the segment next) takes one atomic: it first tries
+// (epoch, n, n - 1) -> (epoch, n, n); a lone CTA (n = 1) swaps its finished word in directly.
+__device__ __forceinline__ bool word_clean(unsigned long long w) {
+  const uint32_t on = (uint32_t)(w >> 16) & 0xFFFFu, oc = (uint32_t)w & 0xFFFFu;
+  return w == 0ull || (on >= 1u && on <= (uint32_t)kMaxCtas && oc == on);
+}
+__device__ bool seg_arrive(unsigned long long* word, uint32_t epoch, uint32_t n, int32_t* dev_status) {
+  const unsigned long long tag = ((unsigned long long)epoch << 32) | ((unsigned long long)n << 16);
+  if (n == 1) {
+    if (!word_clean(atomicExch(word, tag | 1ull))) raise_status(dev_status, VARRATE_ERR_CORRUPT);
+    return true;
+  }
+  unsigned long long old = atomicCAS(word, tag | (n - 1), tag | n);
+  if (old == (tag | (n - 1))) return true;
+  for (int tries = 0; tries < (1 << 16); ++tries) {   // one retry per concurrent arrival
+    const uint32_t oe = (uint32_t)(old >> 32), on = (uint32_t)(old >> 16) & 0xFFFFu;
+    const uint32_t oc = (uint32_t)old & 0xFFFFu;
+    const bool counting = oe == epoch && oc < on;
+    const bool bad = counting ? on != n : !word_clean(old);
+    const unsigned long long nw = (counting && !bad) ? old + 1ull : (tag | 1ull);
+    const unsigned long long prev = atomicCAS(word, old, nw);
+    if (prev == old) {
+      if (bad) raise_status(dev_status, VARRATE_ERR_CORRUPT);
+      return (uint32_t)(nw & 0xFFFFull) == n;
+    }
+    old = prev;
+  }
+  raise_status(dev_status, VARRATE_ERR_TIMEOUT);
+  return false;
+}
+
 struct CombSmem {   // aliases the ring while the last CTA of a segment combines it
   alignas(128) __nv_bfloat16 us[kHeadDim * kHeadDim];   // U_V[g], row j (one bulk copy)
   float ot[kHeadsPad][kHeadDim + 8];                    // merged o~ per head
@@ -422,7 +462,8 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
                   const __nv_bfloat16* __restrict__ basis_v, const __nv_bfloat16* __restrict__ qin,
                   const __nv_bfloat16* __restrict__ tail_k, const __nv_bfloat16* __restrict__ tail_v,
                   int n_tail, __nv_bfloat16* __restrict__ out, float* __restrict__ part,
-                  int* __restrict__ seg_done, int32_t* __restrict__ dev_status, Shape s, int layer) {
+                  unsigned long long* __restrict__ seg_done, int32_t* __restrict__ dev_status, Shape s,
+                  int layer, uint32_t epoch) {
   extern __shared__ __align__(128) unsigned char smem[];
   unsigned char* ring = smem;                                     // NW * ST * STAGE
   static_assert((NW * ST * STAGE) % 16 == 0, "SegSmem must start 16-byte aligned");
@@ -464,7 +505,12 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
   __syncthreads();
   uint32_t n_issued = 0;   // chunks this warp has consumed (== index of its next chunk)
   int n_pending = 0;       // chunks issued but not yet consumed
-  bool timed_out = false;
+  bool timed_out = false;  // this thread saw a bounded wait give up
+  // CTA-uniform: some wait of this CTA gave up, so bulk copies may still be landing in the ring.
+  // From then on nothing writes the ring (merge and combine buffers alias it) and nothing streams;
+  // the CTA still writes an empty partial and arrives on every segment it covers, so the counts of
+  // the other CTAs stay consistent.
+  bool dead = false;
   uint32_t n_comb = 0;     // combines done by this CTA (phase of bar_comb)
   // Cost line: sequence b holds G segments of kSegCost + W_b elements each (W_b > 0), the set-up
   // allowance first. segP = exclusive prefix over sequences (B <= 64: two per lane).
@@ -570,7 +616,7 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
 #pragma unroll
       for (int t = 0; t < kHeadDim / 16; ++t) oacc[t][0] = oacc[t][1] = oacc[t][2] = oacc[t][3] = 0.f;
 
-      const int total = sm.it_pref[kMaxR + 1];
+      const int total = dead ? 0 : sm.it_pref[kMaxR + 1];
       Prod pr;
       pr.k = warp; pr.phase = 0; pr.jc = 0;
       if (pr.k < total) pr.item = item_at(sm, pr.k);
@@ -749,9 +795,13 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
         cons_k += NW;
         if (cons_k < total) cons = item_at(sm, cons_k);
       }
-      // drain: never leave bulk copies in flight into this ring
-      while (n_pending > 0) {
-        mbar_wait_bounded(&bars[n_issued % ST], (n_issued / ST) & 1u, kWaitTries);
+      // drain: never leave bulk copies in flight into this ring (a copy whose wait gave up stays
+      // counted in n_pending and is waited for once more before the CTA exits)
+      while (n_pending > 0 && !timed_out) {
+        if (!mbar_wait_bounded(&bars[n_issued % ST], (n_issued / ST) & 1u, kWaitTries)) {
+          timed_out = true;
+          break;
+        }
         ++n_issued;
         --n_pending;
       }
@@ -762,19 +812,21 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
       for (int e = 0; e < 2; ++e)
 #pragma unroll
         for (int o = 4; o < 32; o <<= 1) Ls[e] += __shfl_xor_sync(0xffffffffu, Ls[e], o);
-      __syncthreads();   // every warp has finished this segment
-      if (g8 == 0) {
+      dead = __syncthreads_or(dead || timed_out);   // every warp has finished this segment
+      if (!dead && g8 == 0) {
         mg.M[warp][2 * c] = Mx[0]; mg.M[warp][2 * c + 1] = Mx[1];
         mg.L[warp][2 * c] = Ls[0]; mg.L[warp][2 * c + 1] = Ls[1];
       }
+      if (!dead) {
 #pragma unroll
-      for (int t = 0; t < kHeadDim / 16; ++t) {
-        mg.acc[warp][2 * c][t * 16 + g8] = oacc[t][0];
-        mg.acc[warp][2 * c + 1][t * 16 + g8] = oacc[t][1];
-        mg.acc[warp][2 * c][t * 16 + g8 + 8] = oacc[t][2];
-        mg.acc[warp][2 * c + 1][t * 16 + g8 + 8] = oacc[t][3];
+        for (int t = 0; t < kHeadDim / 16; ++t) {
+          mg.acc[warp][2 * c][t * 16 + g8] = oacc[t][0];
+          mg.acc[warp][2 * c + 1][t * 16 + g8] = oacc[t][1];
+          mg.acc[warp][2 * c][t * 16 + g8 + 8] = oacc[t][2];
+          mg.acc[warp][2 * c + 1][t * 16 + g8 + 8] = oacc[t][3];
+        }
       }
-      if (tid < kHeadsPad) {
+      if (!dead && tid < kHeadsPad) {
         const int h = tid;
         float mx = -INFINITY, l = 0.f;
 #pragma unroll
@@ -796,34 +848,34 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
       for (int i = tid; i < kHeadsPad * kHeadDim; i += blockDim.x) {
         const int h = i / kHeadDim, j = i % kHeadDim;
         float o = 0.f;
+        if (!dead) {
 #pragma unroll
-        for (int w = 0; w < NW; ++w) o = fmaf(mg.acc[w][h][j], mg.F[w][h], o);
+          for (int w = 0; w < NW; ++w) o = fmaf(mg.acc[w][h][j], mg.F[w][h], o);
+        }
         pout[h * kPartStride + j] = o;
-        if (j == 0) { pout[h * kPartStride + kHeadDim] = mg.mx[h]; pout[h * kPartStride + kHeadDim + 1] = mg.l[h]; }
+        if (j == 0) {   // an abandoned CTA contributes an empty partial
+          pout[h * kPartStride + kHeadDim] = dead ? -INFINITY : mg.mx[h];
+          pout[h * kPartStride + kHeadDim + 1] = dead ? 0.f : mg.l[h];
+        }
       }
       // the last CTA to finish this segment merges every partial of it
       __syncthreads();
       if (tid == 0) {
         __threadfence();
-        const unsigned done = (unsigned)atomicAdd(&seg_done[seg], 1);
-        last_cta = done == (unsigned)(c1 - c0);
-        // every CTA of the segment has counted: zero again for the next call on this workspace
-        if (last_cta) {
-          seg_done[seg] = 0;
-          __threadfence();   // the other CTAs' partials (published before their count) are read next
-        } else if (done > (unsigned)(c1 - c0)) {
-          raise_status(dev_status, VARRATE_ERR_CORRUPT);
-        }
+        last_cta = seg_arrive(&seg_done[seg], epoch, (uint32_t)(c1 - c0 + 1), dev_status);
+        if (last_cta) __threadfence();   // the other CTAs' partials (published before they arrived) are read next
       }
       __syncthreads();
-      if (last_cta) {
+      if (last_cta && !dead) {
         if (!combine_segment(*reinterpret_cast<CombSmem*>(ring), &bar_comb, n_comb & 1u, part, c0, c1, seg,
                              qin + ((long long)b * s.H + (long long)g * s.grp) * kHeadDim,
                              basis_v + ((long long)layer * s.G + g) * kHeadDim * kHeadDim,
                              n_tail ? tail_k + ((long long)b * s.G + g) * n_tail * kHeadDim : nullptr,
                              n_tail ? tail_v + ((long long)b * s.G + g) * n_tail * kHeadDim : nullptr, n_tail,
-                             out + ((long long)b * s.H + (long long)g * s.grp) * kHeadDim, s.grp, tid))
+                             out + ((long long)b * s.H + (long long)g * s.grp) * kHeadDim, s.grp, tid)) {
           timed_out = true;
+          dead = true;   // CTA-uniform: the U_V copy of the combine may still be landing
+        }
         ++n_comb;
       }
       __syncthreads();
@@ -831,7 +883,7 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
     if (++g == s.G) { ++b; g = 0; }
     while (b < s.B && segW[b] == 0) ++b;
     more = b < s.B && seg_start(b, g) < hi_g;
-    if (more) {
+    if (more && !dead) {
       for (int i = tid; i < NW * ST * STAGE / 16; i += blockDim.x)
         reinterpret_cast<uint4*>(ring)[i] = make_uint4(0, 0, 0, 0);
       fence_proxy_async_smem();
@@ -839,21 +891,29 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
     }
   }
   // segments with an empty coded stream (tail only): one CTA each, no partials
-  if (n_empty)
+  if (n_empty && !dead)
   for (int b = 0; b < s.B; ++b)
     for (int g = 0; g < s.G; ++g) {
       const long long seg = (long long)b * s.G + g;
-      if (segW[b] != 0 || seg % C != cta) continue;   // CTA-uniform
+      if (segW[b] != 0 || seg % C != cta || dead) continue;   // CTA-uniform
       __syncthreads();
       if (!combine_segment(*reinterpret_cast<CombSmem*>(ring), &bar_comb, n_comb & 1u, part, 0, -1, seg,
                            qin + ((long long)b * s.H + (long long)g * s.grp) * kHeadDim,
                            basis_v + ((long long)layer * s.G + g) * kHeadDim * kHeadDim,
                            n_tail ? tail_k + ((long long)b * s.G + g) * n_tail * kHeadDim : nullptr,
                            n_tail ? tail_v + ((long long)b * s.G + g) * n_tail * kHeadDim : nullptr, n_tail,
-                           out + ((long long)b * s.H + (long long)g * s.grp) * kHeadDim, s.grp, tid))
+                           out + ((long long)b * s.H + (long long)g * s.grp) * kHeadDim, s.grp, tid)) {
         timed_out = true;
+        dead = true;
+      }
       ++n_comb;
     }
+  if (dead) {
+    // last bounded waits for copies that may still be landing in this CTA's shared memory
+    for (; n_pending > 0; --n_pending, ++n_issued)
+      if (!mbar_wait_bounded(&bar_all[warp * ST + n_issued % ST], (n_issued / ST) & 1u, kWaitTries)) break;
+    if (n_comb > 0 && tid == 0) mbar_wait_bounded(&bar_comb, (n_comb - 1) & 1u, kWaitTries);
+  }
   if (timed_out && lane == 0) raise_status(dev_status, VARRATE_ERR_TIMEOUT);
 }
 
@@ -877,8 +937,9 @@ bool decode_mma_supported(const Shape& s, int n_tail, int num_sms) {
 
 int launch_decode_mma(const Shape& s, const varrate_packed& c, const void* basis_k,
                       const void* basis_v, const void* q, int layer, const void* tail_k,
-                      const void* tail_v, int n_tail, void* out, int32_t* dev_status, int* seg_done,
-                      float* part, int num_sms, cudaStream_t st) {
+                      const void* tail_v, int n_tail, void* out, int32_t* dev_status,
+                      unsigned long long* seg_done, float* part, uint32_t epoch, int num_sms,
+                      cudaStream_t st) {
   const size_t smem = decode_mma_smem_bytes();
   cudaFuncSetAttribute(decode_mma_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   // the grid may be scheduled while its predecessor drains (programmatic dependent launch); it
@@ -897,7 +958,7 @@ int launch_decode_mma(const Shape& s, const varrate_packed& c, const void* basis
                      (const int64_t*)c.bucket_base, (const __nv_bfloat16*)basis_k,
                      (const __nv_bfloat16*)basis_v, (const __nv_bfloat16*)q,
                      (const __nv_bfloat16*)tail_k, (const __nv_bfloat16*)tail_v, n_tail,
-                     (__nv_bfloat16*)out, part, seg_done, dev_status, s, layer);
+                     (__nv_bfloat16*)out, part, seg_done, dev_status, s, layer, epoch);
   return 1;
 }
 

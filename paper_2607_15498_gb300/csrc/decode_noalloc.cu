@@ -6,32 +6,40 @@
 // point runs the same decode kernels as varrate_decode_attn, but takes its scratch (the rotated
 // queries and the per-split partial results) from a fixed array in device global memory that the
 // library itself defines, so the caller passes no workspace and nothing is allocated.
+#include <atomic>
+
 #include "common.cuh"
 #include "kernels.h"
 
 namespace {
 
 // Scratch for every call of this entry point on a device. Every GPU that loads the library holds
-// it until the process exits. Calls share it and it keeps the previous call's contents; the decode
-// kernels write every element they later read, so nothing has to be cleared between calls.
+// it until the process exits. Calls share it and it keeps the previous call's contents. It starts
+// zero-filled (as a __device__ array without initialiser is); its first part holds the decode
+// kernel's completion words, which each call leaves in a finished state (or re-arms, raising
+// VARRATE_ERR_CORRUPT once, if an earlier call overlapped it or gave up), and the decode kernels
+// write every other element they later read, so nothing has to be cleared between calls.
 constexpr size_t kScratchBytes = size_t(4) << 20;   // 4 MiB
 static __device__ __align__(256) unsigned char g_decode_scratch[kScratchBytes];
 
 constexpr int kMaxDevices = 64;
-void* g_scratch_ptr[kMaxDevices] = {nullptr};
+std::atomic<void*> g_scratch_ptr[kMaxDevices];
 
-// Device address of the scratch array on the current device, looked up once per device. In host
-// code the symbol is only a host-side handle, never a device address, so it must not be passed to
-// a kernel directly.
+// Device address of the scratch array on the current device, looked up once per device (with that
+// device current) and cached. In host code the symbol is only a host-side handle, never a device
+// address, so it must not be passed to a kernel directly. Two threads may both look it up the first
+// time; they find the same address. The cache is not told about cudaDeviceReset: after a reset of
+// the device the cached address is stale and this entry point must not be used again in the
+// process.
 void* scratch_on_current_device() {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
-  if (g_scratch_ptr[dev] == nullptr) {
-    void* p = nullptr;
-    if (cudaGetSymbolAddress(&p, g_decode_scratch) != cudaSuccess) return nullptr;
-    g_scratch_ptr[dev] = p;
+  void* p = g_scratch_ptr[dev].load(std::memory_order_acquire);
+  if (p == nullptr) {
+    if (cudaGetSymbolAddress(&p, g_decode_scratch) != cudaSuccess || p == nullptr) return nullptr;
+    g_scratch_ptr[dev].store(p, std::memory_order_release);
   }
-  return g_scratch_ptr[dev];
+  return p;
 }
 
 }  // namespace

@@ -1,5 +1,7 @@
 // Host-side TMA tensor maps (cuTensorMapEncodeTiled reached through the runtime's driver entry
 // point, so the library does not link libcuda directly).
+#include <atomic>
+
 #include <cudaTypedefs.h>
 
 #include "common.cuh"
@@ -8,7 +10,9 @@
 namespace vr {
 
 bool make_tmap_rows_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint32_t box_rows) {
-  static PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
+  // driver entry point, looked up once per process (every thread that looks it up finds the same)
+  static std::atomic<PFN_cuTensorMapEncodeTiled_v12000> cached{nullptr};
+  PFN_cuTensorMapEncodeTiled_v12000 encode = cached.load(std::memory_order_acquire);
   if (encode == nullptr) {
     void* fn = nullptr;
     cudaDriverEntryPointQueryResult q;
@@ -17,6 +21,7 @@ bool make_tmap_rows_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint
         q != cudaDriverEntryPointSuccess || fn == nullptr)
       return false;
     encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    cached.store(encode, std::memory_order_release);
   }
   // [rows][128] bf16, row-major; boxes of 64 columns (128 B, one swizzle span) x box_rows rows
   const cuuint64_t dims[2] = {(cuuint64_t)kHeadDim, (cuuint64_t)rows};

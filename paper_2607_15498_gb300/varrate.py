@@ -256,7 +256,7 @@ class PackedCache:
 
 
 def workspace(cfg: varrate_config, which_call: int, device="cuda") -> torch.Tensor:
-    """Device scratch for one kind of call, zero-filled (decode needs zeros before its first call
-    and leaves its completion counters at zero after each one)."""
+    """Device scratch for one kind of call, zero-filled (decode needs its completion words zero
+    before the first call that uses them; every call leaves them finished for the next one)."""
     n = varrate_workspace_bytes(cfg, which_call)
     return torch.zeros(max(n, 256), dtype=torch.uint8, device=device)

@@ -10,8 +10,9 @@ one from host copies of the same tensors."""
 import numpy as np
 import pytest
 
-from gpu_helpers import (O, V, cfg_for, coef_tol, decode_tol, f64, gpu_decode, gpu_encode,
-                         gpu_pack, oracle_layer, salience_close, synth, unpack)
+from gpu_helpers import (O, V, cfg_for, coef_tol, decode_close, decode_errors, f64, gpu_decode,
+                         gpu_encode, gpu_pack, oracle_layer, salience_close, synth, unpack,
+                         uniform_weight_output)
 
 pytestmark = pytest.mark.gpu
 
@@ -49,18 +50,23 @@ def _check_encode(run):
 
 
 def _check_decode(run, n_steps=2):
+    """Decode of the sampled pairs within the per-row relative bar; at the same size a score-blind
+    output (uniform weights) must fail that bar, so the check is able to catch a wrong kernel."""
     wl, cfg, r = run["wl"], run["cfg"], run["gpu"]
     _, _, _, bk, bv = run["inputs"]
-    worst = 0.0
+    worst = (0.0, 0.0)
     for (b, l), ref in run["refs"].items():
         qs = synth.stack_decode_queries(wl, l, n_steps)
+        blind = uniform_weight_output(ref, f64(bv[l]), wl.group)
         for step in range(n_steps):
             out, st = gpu_decode(cfg, r["packed"], bk, bv, qs[step], l)
             assert st == V.OK
             want = O.decode_coef(f64(qs[step][b]), ref["coef_k"], ref["coef_v"], ref["ranks"],
                                  f64(bk[l]), f64(bv[l]))
-            worst = max(worst, float(np.abs(out[b] - want).max()))
-    assert worst <= decode_tol(cfg), worst
+            assert decode_close(out[b], want, cfg), (b, l, step, decode_errors(out[b], want))
+            assert not decode_close(blind, want, cfg), (b, l, step, decode_errors(blind, want))
+            worst = tuple(max(a, e) for a, e in zip(worst, decode_errors(out[b], want)))
+    print(f"N={wl.n_ctx}: decode worst relative / absolute error {worst[0]:.3e} / {worst[1]:.3e}")
 
 
 def _check_pack(run, n_tokens=4096):
