@@ -196,7 +196,7 @@ varrate_status varrate_encode(const varrate_config* cfg, const void* q_win, cons
  *           action by the caller; results written while the words were inconsistent are not to be
  *           trusted. Replaying a captured launch of this call is fine: the replay keeps its tag and
  *           finds its own finished words.
- * Kernels: in bf16 with n_tail <= 64, batch <= 64 and batch * n_kv_heads <= 4096 one fused kernel
+ * Kernels: in bf16 with n_tail <= 256, batch <= 64 and batch * n_kv_heads <= 4096 one fused kernel
  * runs. It is launched with programmatic stream serialization and allows the next kernel on
  * `stream` to be scheduled while it runs: a following kernel launched with that attribute must wait
  * for it (griddepcontrol.wait / cudaGridDependencySynchronize) before it reads `out` or

@@ -326,21 +326,27 @@ __device__ bool seg_arrive(unsigned long long* word, uint32_t epoch, uint32_t n,
   return false;
 }
 
+constexpr int kMaxTailFused = 256;   // exact tail tokens the fused kernel stages in the ring
+
 struct CombSmem {   // aliases the ring while the last CTA of a segment combines it
-  alignas(128) __nv_bfloat16 us[kHeadDim * kHeadDim];   // U_V[g], row j (one bulk copy)
-  float ot[kHeadsPad][kHeadDim + 8];                    // merged o~ per head
-  float qrow[kHeadsPad][kHeadDim];
-  float tsc[kHeadsPad][64];                             // exact tail scores, then weights (n_tail <= 64)
-  float tmax[kHeadsPad], hl[kHeadsPad];
+  alignas(128) __nv_bfloat16 us[kHeadDim * kHeadDim];       // U_V[g], row j (one bulk copy)
+  alignas(128) __nv_bfloat16 tk[kMaxTailFused * kHeadDim];  // exact tail keys, row t (one bulk copy)
+  alignas(128) __nv_bfloat16 tv[kMaxTailFused * kHeadDim];  // exact tail values, row t (one bulk copy)
+  float ot[kHeadsPad][kHeadDim + 8];                        // merged o~ per head
+  float tsc[kHeadsPad][kMaxTailFused + 8];                  // tail scores, then tail weights
+  float hl[kHeadsPad];                                      // softmax normaliser per head
 };
 static_assert(sizeof(CombSmem) <= (size_t)NW * ST * STAGE, "combine buffers fit in the ring");
 static_assert(NW == kHeadsPad, "one warp per head in the combine");
 
 // Merge the partials of segment (b, g) written by CTAs c0..c1 (slot cc + seg; none if c1 < c0),
-// add the exact tail, rotate back with U_V^T (m16n8k16 tiles, o~ split hi + lo) and normalise.
-// Called by all 256 threads; the ring is idle. Warp h merges head h, lane l columns 4l .. 4l + 3,
-// with the partials of up to 8 CTAs in flight at once (online rescaling across batches).
-// Returns false if the U_V copy timed out.
+// add the exact tail, rotate back with U_V^T and normalise. Called by all 256 threads; the ring
+// is idle. U_V and the tail's keys and values are staged in the ring by bulk copies while the
+// partials are merged (warp h merges head h, lane l columns 4l .. 4l + 3, with the partials of up
+// to 8 CTAs in flight at once). Tail scores are m16n8k16 tiles (16 tail tokens x 8 heads, exact
+// bf16 products of key and query); the tail's values join the rotation as further k-steps:
+//   out^T[col][head] = sum_j U_V[j][col] o~[head][j] + sum_t v_t[col] w[head][t]
+// with o~ and the tail weights w split hi + lo in bf16. Returns false if a staging copy timed out.
 __device__ bool combine_segment(CombSmem& cs, uint64_t* bar, uint32_t parity, const float* __restrict__ part,
                                 int c0, int c1, long long seg, const __nv_bfloat16* __restrict__ q,
                                 const __nv_bfloat16* __restrict__ Uv, const __nv_bfloat16* __restrict__ tail_k,
@@ -348,36 +354,37 @@ __device__ bool combine_segment(CombSmem& cs, uint64_t* bar, uint32_t parity, co
                                 __nv_bfloat16* __restrict__ out, int grp, int tid) {
   const int lane = tid & 31, warp = tid >> 5;
   const int g8 = lane >> 2, c = lane & 3;
-  fence_proxy_async_smem();   // earlier generic accesses of the ring precede the async write
+  const int n_tt = (n_tail + 15) >> 4;   // 16-token tiles of the tail
+  fence_proxy_async_smem();   // earlier generic accesses of the ring precede the async writes
   __syncthreads();
   if (tid == 0) {
-    mbar_arrive_expect_tx(bar, kHeadDim * kHeadDim * 2);
+    const uint32_t tail_bytes = (uint32_t)n_tail * kHeadDim * 2;
+    mbar_arrive_expect_tx(bar, kHeadDim * kHeadDim * 2 + 2 * tail_bytes);
     bulk_g2s(smem_addr(cs.us), Uv, kHeadDim * kHeadDim * 2, bar);
+    if (n_tail) {
+      bulk_g2s(smem_addr(cs.tk), tail_k, tail_bytes, bar);
+      bulk_g2s(smem_addr(cs.tv), tail_v, tail_bytes, bar);
+    }
   }
   __syncwarp();
-  const float scale = kLog2e * rsqrtf((float)kHeadDim);
-  if (n_tail) {                                                   // exact tail scores and maxima
-    for (int i = tid; i < grp * kHeadDim; i += blockDim.x) cs.qrow[i / kHeadDim][i % kHeadDim] = __bfloat162float(q[i]);
-    __syncthreads();
-    for (int i = warp; i < grp * n_tail; i += NW) {
-      const int h = i / n_tail, t = i % n_tail;
-      const __nv_bfloat16* tk = tail_k + (long long)t * kHeadDim;
-      float a = 0.f;
-#pragma unroll
-      for (int k = 0; k < 4; ++k) a = fmaf(cs.qrow[h][lane * 4 + k], __bfloat162float(tk[lane * 4 + k]), a);
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) a += __shfl_xor_sync(0xffffffffu, a, o);
-      if (lane == 0) cs.tsc[h][t] = a * scale;
-    }
-    __syncthreads();
+  // rows of the last tail tile past n_tail read as zeros (disjoint from the copies' bytes)
+  for (int i = n_tail * kHeadDim + tid; i < n_tt * 16 * kHeadDim; i += blockDim.x) {
+    cs.tk[i] = __float2bfloat16_rn(0.f);
+    cs.tv[i] = __float2bfloat16_rn(0.f);
   }
+  // query B fragments of the tail scores: B[k][n] = q[head n][k], pairs of k per register
+  uint32_t qb[kHeadDim / 16][2];
+#pragma unroll
+  for (int ks = 0; ks < kHeadDim / 16; ++ks) {
+    const __nv_bfloat16* qr = q + (long long)(g8 < grp ? g8 : 0) * kHeadDim + ks * 16 + 2 * c;
+    qb[ks][0] = g8 < grp && n_tail ? *reinterpret_cast<const uint32_t*>(qr) : 0u;
+    qb[ks][1] = g8 < grp && n_tail ? *reinterpret_cast<const uint32_t*>(qr + 8) : 0u;
+  }
+  // merge the partials of the coded stream
   const int h = warp;
   float M = -INFINITY, L = 0.f;
   float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
   if (h < grp) {
-    for (int t = lane; t < n_tail; t += 32) M = fmaxf(M, cs.tsc[h][t]);
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
     const int np = c1 - c0 + 1;
     for (int cb = 0; cb < np; cb += 8) {
       float m[8], l[8];
@@ -410,31 +417,62 @@ __device__ bool combine_segment(CombSmem& cs, uint64_t* bar, uint32_t parity, co
         M = mx;
       }
     }
-    float lt = 0.f;                                               // tail weights at the final max
-    for (int t = lane; t < n_tail; t += 32) {
-      const float w = exp2f(cs.tsc[h][t] - M);
-      cs.tsc[h][t] = w;
+  }
+  if (!__syncthreads_and(mbar_wait_bounded(bar, parity, kWaitTries))) return false;
+  __syncwarp();
+  // exact tail scores (log2 units): warp w takes tail tiles w, w + 8, ...
+  const float scale = kLog2e * rsqrtf((float)kHeadDim);
+  for (int tt = warp; tt < n_tt; tt += NW) {
+    float sc[4] = {0.f, 0.f, 0.f, 0.f};
+    const int row = tt * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
+#pragma unroll
+    for (int ks = 0; ks < kHeadDim / 16; ++ks) {
+      uint32_t a[4];
+      ldsm_x4(smem_addr(&cs.tk[row * kHeadDim + ks * 16 + (lane >> 4) * 8]), a);
+      mma_bf16_16816(sc, a, qb[ks][0], qb[ks][1]);
+    }
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {   // rows tt*16 + g8 (+8), heads 2c, 2c+1
+      const int t = tt * 16 + g8 + (e >> 1) * 8;
+      cs.tsc[2 * c + (e & 1)][t] = t < n_tail ? sc[e] * scale : -INFINITY;
+    }
+  }
+  __syncthreads();
+  // per head: fold the tail into the softmax, tail weights in place of the scores
+  {
+    float tm = -INFINITY;
+    if (h < grp)
+      for (int t = lane; t < n_tail; t += 32) tm = fmaxf(tm, cs.tsc[h][t]);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) tm = fmaxf(tm, __shfl_xor_sync(0xffffffffu, tm, o));
+    const float mx = fmaxf(M, tm);
+    const float f = (M == -INFINITY || mx == -INFINITY) ? 0.f : exp2f(M - mx);
+    acc.x *= f; acc.y *= f; acc.z *= f; acc.w *= f;
+    float lt = 0.f;
+    for (int t = lane; t < n_tt * 16; t += 32) {
+      const float w = (h < grp && t < n_tail) ? exp2f(cs.tsc[h][t] - mx) : 0.f;
+      cs.tsc[h][t] = w;   // zero for padded heads and rows past the tail
       lt += w;
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) lt += __shfl_xor_sync(0xffffffffu, lt, o);
-    if (lane == 0) cs.hl[h] = L + lt;
+    if (lane == 0) cs.hl[h] = L * f + lt;
+    if (h >= grp) acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    *reinterpret_cast<float4*>(&cs.ot[h][4 * lane]) = acc;     // zero for padded heads
   }
-  *reinterpret_cast<float4*>(&cs.ot[h][4 * lane]) = acc;        // zero for padded heads
-  if (!__syncthreads_and(mbar_wait_bounded(bar, parity, kWaitTries))) return false;
-  __syncwarp();
-  // out^T[col][head] = sum_j U_V[j][col] o~[head][j]: warp w owns columns 16w .. 16w + 15
+  __syncthreads();
+  // out^T[col][head]: warp w owns columns 16w .. 16w + 15
   {
-    // four independent accumulators (hi / lo part of o~, even / odd k-step) keep the chain of
-    // dependent MMAs four deep instead of sixteen
+    // four independent accumulators (hi / lo part of the B operand, even / odd k-step) keep the
+    // chain of dependent MMAs short
     float d[4][4] = {};
     const int col0 = warp * 16;
+    const int col = col0 + ((lane >> 3) & 1) * 8;
+    const int jr = (lane & 7) + ((lane >> 4) & 1) * 8;
 #pragma unroll
     for (int ks = 0; ks < kHeadDim / 16; ++ks) {
-      const int j = ks * 16 + (lane & 7) + ((lane >> 4) & 1) * 8;
-      const int col = col0 + ((lane >> 3) & 1) * 8;
       uint32_t a[4];
-      ldsm_x4_trans(smem_addr(&cs.us[j * kHeadDim + col]), a);
+      ldsm_x4_trans(smem_addr(&cs.us[(ks * 16 + jr) * kHeadDim + col]), a);
       const int jb = ks * 16 + 2 * c;
       uint32_t h0, l0, h1, l1;
       split_bf16(cs.ot[g8][jb], cs.ot[g8][jb + 1], h0, l0);
@@ -442,14 +480,27 @@ __device__ bool combine_segment(CombSmem& cs, uint64_t* bar, uint32_t parity, co
       mma_bf16_16816(d[ks & 1], a, h0, h1);
       mma_bf16_16816(d[2 + (ks & 1)], a, l0, l1);
     }
+    for (int ts = 0; ts < n_tt; ts += 2) {   // the tail's values, 16 tokens per k-step
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        if (ts + u < n_tt) {
+          uint32_t a[4];
+          ldsm_x4_trans(smem_addr(&cs.tv[((ts + u) * 16 + jr) * kHeadDim + col]), a);
+          const int tb = (ts + u) * 16 + 2 * c;
+          uint32_t h0, l0, h1, l1;
+          split_bf16(cs.tsc[g8][tb], cs.tsc[g8][tb + 1], h0, l0);
+          split_bf16(cs.tsc[g8][tb + 8], cs.tsc[g8][tb + 9], h1, l1);
+          mma_bf16_16816(d[u], a, h0, h1);
+          mma_bf16_16816(d[2 + u], a, l0, l1);
+        }
+      }
+    }
 #pragma unroll
     for (int e = 0; e < 4; ++e) {
-      const int col = col0 + g8 + (e >> 1) * 8, hh = 2 * c + (e & 1);
+      const int oc = col0 + g8 + (e >> 1) * 8, hh = 2 * c + (e & 1);
       if (hh < grp) {
-        float y = (d[0][e] + d[1][e]) + (d[2][e] + d[3][e]);
-        for (int t = 0; t < n_tail; ++t)
-          y = fmaf(cs.tsc[hh][t], __bfloat162float(tail_v[(long long)t * kHeadDim + col]), y);
-        out[(long long)hh * kHeadDim + col] = __float2bfloat16_rn(y / cs.hl[hh]);
+        const float y = (d[0][e] + d[1][e]) + (d[2][e] + d[3][e]);
+        out[(long long)hh * kHeadDim + oc] = __float2bfloat16_rn(y / cs.hl[hh]);
       }
     }
   }
@@ -931,7 +982,7 @@ bool decode_mma_supported(const Shape& s, int n_tail, int num_sms) {
   // the cost line (at most B G cap elements) times the grid size must stay below 2^62
   const unsigned long long line = (unsigned long long)s.B * s.G * ((unsigned long long)s.cap + kSegCost);
   return s.dtype == VARRATE_BF16 && s.B <= 64 && (long long)s.B * s.G <= kDecodeMaxSegs &&
-         n_tail <= 64 && num_sms >= 1 && num_sms <= kMaxCtas &&
+         n_tail <= kMaxTailFused && num_sms >= 1 && num_sms <= kMaxCtas &&
          line <= (1ull << 62) / (unsigned long long)num_sms;
 }
 

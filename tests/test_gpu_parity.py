@@ -218,13 +218,22 @@ def test_decode_matches_oracle(inputs, name):
     _decode_check(CASES[name], inputs[name])
 
 
-def test_decode_with_exact_tail(inputs):
-    _decode_check(CASES["llama_ragged"], inputs["llama_ragged"], n_tail=37, n_steps=2)
+@pytest.mark.parametrize("n_tail", [1, 37, 160, 256])
+def test_decode_with_exact_tail(inputs, n_tail):
+    # the fused bf16 kernel stages up to 256 tail tokens (160 = a 32-token window plus 128 decode
+    # steps appended after the cache)
+    _decode_check(CASES["llama_ragged"], inputs["llama_ragged"], n_tail=n_tail, n_steps=2)
 
 
 def test_decode_with_long_exact_tail(inputs):
-    # more than 64 tail tokens: the bf16 call takes the general split-and-combine kernels
-    _decode_check(CASES["llama_ragged"], inputs["llama_ragged"], n_tail=100, n_steps=1)
+    # more than 256 tail tokens: the bf16 call takes the general split-and-combine kernels
+    _decode_check(CASES["llama_ragged"], inputs["llama_ragged"], n_tail=300, n_steps=1)
+
+
+def test_decode_tail_only(inputs):
+    """Empty coded set: the whole context is the exact window, plus an exact tail."""
+    wl = synth.workload("llama1", n_kv_heads=2, n_ctx=32, window=32, batch=2)
+    _decode_check(wl, synth.stack_inputs(wl), n_tail=45, n_steps=1)
 
 
 def test_decode_uniform_mode(inputs):

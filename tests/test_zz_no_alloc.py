@@ -6,7 +6,7 @@ varrate_decode_attn_noalloc takes its scratch from a fixed array inside the libr
 same kernels as varrate_decode_attn with the same grid and merge order, so its output must equal,
 bit for bit, that of a call with caller workspace, on two calls in a row (the array is reused and
 keeps the previous call's contents). Covered: the fused bf16 kernel (no tail), the general bf16
-kernels (a 100-token exact tail) and the fp32 kernels, which place their scratch differently.
+kernels (a 300-token exact tail) and the fp32 kernels, which place their scratch differently.
 Collected last, so that a run stopping at the first failure has already run every other test."""
 import numpy as np
 import pytest
@@ -19,7 +19,7 @@ def _cases():
     import synth
     return {
         "bf16_fused": (synth.workload("llama1", n_kv_heads=4, n_ctx=6000 + 13, batch=2, n_layers=2), 0),
-        "bf16_long_tail": (synth.workload("llama1", n_kv_heads=2, n_ctx=3000 + 7, batch=2, n_layers=2), 100),
+        "bf16_long_tail": (synth.workload("llama1", n_kv_heads=2, n_ctx=3000 + 7, batch=2, n_layers=2), 300),
         "f32": (synth.workload("tiny", n_kv_heads=2, group=2, n_ctx=999, window=7, n_layers=2), 5),
     }
 
