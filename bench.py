@@ -135,6 +135,18 @@ class Clocks:
 
 # ------------------------------------------------------------------------ our CUDA path
 
+def capture(fn):
+    """The calls fn() issues, captured once into a CUDA graph (fn must take its stream from
+    torch's current stream); replaying it launches the same kernels with the same arguments
+    without the host's per-call cost, as a serving loop that captures its decode step would."""
+    g = torch.cuda.CUDAGraph()
+    torch.cuda.synchronize()
+    with torch.cuda.graph(g):
+        fn()
+    torch.cuda.synchronize()
+    return g
+
+
 def algorithmic_decode_bytes(packed, cfg, elem=2):
     """Bytes one decode call (one layer, all sequences) must move: K and V coefficients
     (sum of ranks, no padding) of every head, the two bases, queries and outputs."""
@@ -172,11 +184,21 @@ def run_ours(args, wl, rank, world):
         V.check(V.varrate_encode(cfg, qw, k, v, bk, bv, None, packed, realized, status, ws_enc,
                                  stream), "varrate_encode")
 
-    def decode_phase():
+    def decode_calls():
         for s in range(D):
             for l in range(L):
                 V.check(V.varrate_decode_attn(cfg, packed, bk, bv, qdec[s, l], l, None, None, 0,
-                                              out, status, ws_dec, stream), "varrate_decode_attn")
+                                              out, status, ws_dec, None), "varrate_decode_attn")
+
+    decode_calls()                      # first calls on this workspace and device: outside capture
+    torch.cuda.synchronize()
+    graph = None if args.no_graph else capture(decode_calls)
+
+    def decode_phase():
+        if graph is None:
+            decode_calls()
+        else:
+            graph.replay()
 
     for _ in range(args.warmup):
         encode()
@@ -357,15 +379,21 @@ def sweep_config(V, wl, dev, peak, stream, decode_steps, copies=1, flush=False, 
             for l in range(wl.n_layers):
                 V.check(V.varrate_decode_attn(cfg, caches[(s_ * wl.n_layers + l) % copies], bk, bv,
                                               qdec[s_, l], l, None, None, 0, out, status, ws_dec,
-                                              stream), "varrate_decode_attn")
+                                              None), "varrate_decode_attn")
     phase(min(decode_steps, 3))
+    g = capture(lambda: phase(decode_steps))
+    g.replay()
     torch.cuda.synchronize()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    phase(decode_steps)
-    e1.record(stream)
-    torch.cuda.synchronize()
-    dec_ms = e0.elapsed_time(e1)
+    times = []
+    for _ in range(3):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        g.replay()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        times.append(e0.elapsed_time(e1))
+    dec_ms = statistics.median(times)
+    del g
     dec_status = int(status.item())
     n_calls = decode_steps * wl.n_layers
     dec_bytes = decode_steps * (sum(per_layer) + wl.n_layers * fixed)
@@ -378,6 +406,8 @@ def sweep_config(V, wl, dev, peak, stream, decode_steps, copies=1, flush=False, 
            "decode_us_per_layer_call": round(dec_ms * 1e3 / n_calls, 2),
            "decode_bytes_per_layer_call": int(dec_bytes / n_calls),
            "decode_status": V.status_string(dec_status), "decode_steps": decode_steps,
+           "decode_issue": "CUDA graph of the decode steps (one captured call per layer and step), "
+                           "median of 3 replays",
            "l2": (f"{copies} packed copies cycled ({copies * int(sum(per_layer) / wl.n_layers / 1e6)} MB per "
                   f"cycle of layer calls > L2)") if copies > 1 else
                  "all layers' packed caches read per step (> L2)",
@@ -431,18 +461,24 @@ def sweep_reuse(V, wl, dev, peak, stream, n_batches, n_window, n_decode):
         # the tail of step i is the first i + 1 rows: one contiguous [B][G][i + 1][d] block per layer
         tails = [[(tk[l, :, :, : i + 1].contiguous(), tv[l, :, :, : i + 1].contiguous())
                   for l in range(wl.n_layers)] for i in range(n_steps)]
-        torch.cuda.synchronize()
+        def window(lo, hi):
+            for i in range(lo, hi):
+                for l in range(wl.n_layers):
+                    a, b_ = tails[i][l]
+                    V.check(V.varrate_decode_attn(cfg, packed, bk, bv, q[i, l], l, a, b_, i + 1,
+                                                  out, status, ws_dec, None), "varrate_decode_attn")
+        if qb == 0:
+            window(0, n_steps)          # first calls on this workspace: outside capture
+        gw = capture(lambda: window(0, n_window))
+        gd = capture(lambda: window(n_window, n_steps))
         ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
         ev[0].record(stream)
-        for i in range(n_steps):
-            if i == n_window:
-                ev[1].record(stream)
-            for l in range(wl.n_layers):
-                a, b_ = tails[i][l]
-                V.check(V.varrate_decode_attn(cfg, packed, bk, bv, q[i, l], l, a, b_, i + 1, out,
-                                              status, ws_dec, stream), "varrate_decode_attn")
+        gw.replay()
+        ev[1].record(stream)
+        gd.replay()
         ev[2].record(stream)
         torch.cuda.synchronize()
+        del gw, gd
         if qb > 0:
             total_ms += ev[0].elapsed_time(ev[2])
             win_ms.append(ev[0].elapsed_time(ev[1]))
@@ -462,6 +498,8 @@ def sweep_reuse(V, wl, dev, peak, stream, n_batches, n_window, n_decode):
             "window_ms_per_batch": round(statistics.mean(win_ms), 3),
             "ms_per_query_batch": round(total_ms / n_batches, 3),
             "decode_status": V.status_string(int(status.item())),
+            "decode_issue": "per query batch, CUDA graphs of its window steps and of its decode "
+                            "steps (one captured call per layer and step)",
             "l2": "packed cache of all layers (3.4 GB) read per step (> L2)"}
 
 
@@ -626,6 +664,8 @@ def main():
     ap.add_argument("--no-sweep", action="store_true",
                     help="skip the other seeded configurations (llama1, qwen budget sweep, reuse)")
     ap.add_argument("--reuse-batches", type=int, default=16)
+    ap.add_argument("--no-graph", action="store_true",
+                    help="issue the headline decode calls from the host instead of replaying a graph")
     ap.add_argument("--layers", type=int, default=None, help="override the layer count (profiling)")
     ap.add_argument("--batch", type=int, default=None, help="override the sequence count (profiling)")
     args = ap.parse_args()
@@ -642,6 +682,8 @@ def main():
                 if wl.name.startswith("llama") else wl.name,
                 "global_batch": wl.batch * world, "seq_len": wl.n_ctx,
                 "decode_steps": args.decode_steps, "parallelism": f"replicas over sequences x{world}",
+                "decode_issue": "host-issued calls" if args.no_graph else
+                                "CUDA graph replay (one captured call per layer and step)",
                 "l2": "inputs larger than L2 (packed cache of all layers re-read every decode step)"}
     base = {"metric": METRIC, "unit": "GB/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,

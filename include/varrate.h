@@ -183,19 +183,17 @@ varrate_status varrate_encode(const varrate_config* cfg, const void* q_win, cons
  *           n_tail == 0); 0 <= n_tail <= 4096 (more is VARRATE_ERR_UNSUPPORTED)
  *   out     [B][H][d]  dtype
  *   ws      at least varrate_workspace_bytes(cfg, VARRATE_CALL_DECODE) bytes, zero-filled before
- *           the first decode call that uses it. Its first 32 KiB hold one 64-bit completion word
- *           per (sequence, KV head) (at most 4096): the tag of the last call that used it, the
- *           number of thread blocks that call split the pair over, and how many have finished.
- *           Every call leaves its words finished; the rest of the workspace is scratch that a call
- *           writes before it reads. So one workspace serves any number of later decode calls (any
- *           shape), provided they are ordered on one stream. Calls that overlap on one workspace
- *           (different streams, host threads) race and give wrong results. A call that finds a
- *           word that is neither zero nor finished (an overlapping call, a call that gave up with
- *           VARRATE_ERR_TIMEOUT, or garbage) raises VARRATE_ERR_CORRUPT in *dev_status and re-arms
- *           the word for itself, so the next call on the workspace is clean again without any
- *           action by the caller; results written while the words were inconsistent are not to be
- *           trusted. Replaying a captured launch of this call is fine: the replay keeps its tag and
- *           finds its own finished words.
+ *           the first decode call that uses it. Its first 33024 bytes are a header kept by the
+ *           fused kernel (below): a count of its calls on this workspace and two alternating sets
+ *           of per-(sequence, KV head) arrival counters (at most 4096 pairs). A call counts on the
+ *           set of its call count's parity and clears the other set for the next call; the rest of
+ *           the workspace is scratch that a call writes before it reads. So one workspace serves
+ *           any number of later decode calls (any shape), provided they are ordered on one stream,
+ *           and captured launches can be replayed. Calls that overlap on one workspace (different
+ *           streams, host threads) race and give wrong results. A call that finds counts left by
+ *           an earlier call (an overlapping call, a call that gave up with VARRATE_ERR_TIMEOUT, or
+ *           garbage) raises VARRATE_ERR_CORRUPT in *dev_status; its results are not to be trusted,
+ *           and the next call on the workspace is clean again without any action by the caller.
  * Kernels: in bf16 with n_tail <= 256, batch <= 64 and batch * n_kv_heads <= 4096 one fused kernel
  * runs. It is launched with programmatic stream serialization and allows the next kernel on
  * `stream` to be scheduled while it runs: a following kernel launched with that attribute must wait
@@ -223,10 +221,10 @@ varrate_status varrate_decode_attn(const varrate_config* cfg, const varrate_pack
  *    that device again in the process.
  *  - All calls share the one array: calls that overlap on the GPU (other streams, other host
  *    threads) race on it and must be serialised by the caller. The array starts zero-filled and
- *    keeps the last call's contents: its completion words work as described for
- *    varrate_decode_attn (left finished by every call; after an overlap or a timed-out call the
- *    next call reports VARRATE_ERR_CORRUPT once and re-arms them, since the caller cannot clear
- *    this array), and the rest is written before it is read. */
+ *    keeps the last call's contents: its header works as described for varrate_decode_attn (after
+ *    an overlap or a timed-out call one call reports VARRATE_ERR_CORRUPT and the next is clean
+ *    again, which matters here because the caller cannot clear this array), and the rest is
+ *    written before it is read. */
 varrate_status varrate_decode_attn_noalloc(const varrate_config* cfg, const varrate_packed* cache,
                                            const void* basis_k, const void* basis_v, const void* q,
                                            int32_t layer, const void* tail_k, const void* tail_v,

@@ -73,13 +73,6 @@ int num_sms() {
   return n;
 }
 
-// Tag of one decode call in the workspace's completion words: a process-wide counter, never 0.
-uint32_t next_decode_epoch() {
-  static std::atomic<uint32_t> counter{0};
-  uint32_t e = counter.fetch_add(1, std::memory_order_relaxed) + 1;
-  if (e == 0) e = counter.fetch_add(1, std::memory_order_relaxed) + 1;
-  return e;
-}
 
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
@@ -236,8 +229,9 @@ varrate_status varrate_decode_attn(const varrate_config* cfg, const varrate_pack
   const size_t need = ws_bytes(cfg, VARRATE_CALL_DECODE);
   if (ws_bytes_ < need || ws == nullptr) return VARRATE_ERR_WORKSPACE;
   const Shape s = make_shape(cfg, cache->cap_elems);
-  vr::launch_decode(s, *cache, basis_k, basis_v, q, layer, tail_k, tail_v, n_tail, out, dev_status,
-                    ws, next_decode_epoch(), num_sms(), (cudaStream_t)stream);
+  if (vr::launch_decode(s, *cache, basis_k, basis_v, q, layer, tail_k, tail_v, n_tail, out, dev_status,
+                        ws, num_sms(), (cudaStream_t)stream) < 0)
+    return VARRATE_ERR_CUDA;
   return launched();
 }
 

@@ -275,6 +275,12 @@ namespace vr {
 // Programmatic dependent launch: wait until the preceding grid in the stream has completed and its
 // memory is visible (returns at once when launched without the attribute) / allow the next grid to
 // be scheduled.
+// Atomic add at GPU scope with acquire and release semantics; returns the previous value.
+__device__ __forceinline__ uint32_t atom_add_acq_rel_gpu(uint32_t* p, uint32_t v) {
+  uint32_t old;
+  asm volatile("atom.add.acq_rel.gpu.global.u32 %0, [%1], %2;\n" : "=r"(old) : "l"(p), "r"(v) : "memory");
+  return old;
+}
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;\n" ::: "memory"); }
 __device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory"); }
 }  // namespace vr

@@ -370,13 +370,12 @@ size_t decode_ws_bytes(const Shape& s, int num_sms) {
 int launch_decode(const Shape& s, const varrate_packed& cache, const void* basis_k,
                   const void* basis_v, const void* q, int layer, const void* tail_k,
                   const void* tail_v, int n_tail, void* out, int32_t* dev_status, void* ws,
-                  uint32_t epoch, int num_sms, cudaStream_t st) {
-  // completion words: the first kDecodeCounterBytes of the workspace
-  unsigned long long* seg_done = reinterpret_cast<unsigned long long*>(ws);
+                  int num_sms, cudaStream_t st) {
+  void* header = ws;   // completion counting: the first kDecodeCounterBytes of the workspace
   ws = static_cast<char*>(ws) + kDecodeCounterBytes;
   if (decode_mma_supported(s, n_tail, num_sms))
     return launch_decode_mma(s, cache, basis_k, basis_v, q, layer, tail_k, tail_v, n_tail, out,
-                             dev_status, seg_done, reinterpret_cast<float*>(ws), epoch, num_sms, st);
+                             dev_status, header, reinterpret_cast<float*>(ws), num_sms, st);
   const int S = decode_splits(s, num_sms);
   float* qt = reinterpret_cast<float*>(ws);
   size_t a = (size_t)s.B * s.H * kHeadDim * sizeof(float);

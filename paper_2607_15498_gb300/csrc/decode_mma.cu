@@ -13,10 +13,12 @@
 // short one), each one contiguous block.
 //
 // Memory path. Each warp owns a 3-stage shared-memory ring filled by one 1-D TMA bulk copy per
-// chunk that completes on a per-stage mbarrier; the warp stays 2 chunks ahead of the chunk it
-// computes on, across item boundaries, so loads never wait on arithmetic. The per-row rotation of
-// the 8-slot groups keeps the unpadded staged rows free of shared-memory bank conflicts. Rows >= r of a chunk are never loaded; they are masked out of the tensor-core
-// fragments instead, and the ring only ever holds finite coefficients.
+// chunk that completes on a per-stage mbarrier; while the warp computes on one stage the other
+// two are in flight (the stage it finishes is refilled with the chunk three ahead), across item
+// boundaries, so loads never wait on arithmetic. The per-row rotation of
+// the 8-slot groups keeps the unpadded staged rows free of shared-memory bank conflicts. Rows >= r
+// of a chunk are never loaded: they are masked out of the K and V fragments (not multiplied by
+// zero), so whatever the ring held before never reaches the arithmetic and it is never cleared.
 //
 // Arithmetic (per warp, fp32 accumulate, all operands exact or split hi+lo in bf16):
 //   scores   S^T[slot][head] += K^T[slot][j] * Q~^T[j][head]   (mma m16n8k16; K via ldmatrix.trans,
@@ -33,6 +35,8 @@
 // shuffles, votes and tensor-core fragments: left to itself a diverged warp reaching those
 // instructions was measured to lose thousands of cycles.
 #include <stddef.h>
+
+#include <atomic>
 
 #include "common.cuh"
 #include "kernels.h"
@@ -117,6 +121,14 @@ struct Item {
   int it;   // item index inside the bucket
 };
 
+__device__ __forceinline__ Item item_at(const SegSmem& sm, int k);
+
+// Item k after item x = item k - NW (round-robin): NW further in the same bucket, else a search.
+__device__ __forceinline__ Item next_rr(const SegSmem& sm, Item x, int k) {
+  if (k < sm.it_pref[x.r + 1]) { x.it += NW; return x; }
+  return item_at(sm, k);
+}
+
 __device__ __forceinline__ Item item_at(const SegSmem& sm, int k) {
   int lo = 0, hi = kMaxR + 1;   // it_pref[lo] <= k < it_pref[hi]
   while (hi - lo > 1) {
@@ -149,8 +161,7 @@ struct Prod {
 // Returns false (and issues nothing) when the stream is exhausted.
 __device__ __forceinline__ bool issue_chunk(Prod& p, const SegSmem& sm, const __nv_bfloat16* cK,
                                             const __nv_bfloat16* cV, uint32_t stage_addr,
-                                            uint64_t* bar, int total, int lane, uint64_t policy,
-                                            bool fence = true) {
+                                            uint64_t* bar, int total, int lane, uint64_t policy) {
   if (p.k >= total) return false;
   const int r = p.item.r;
   const long long n8 = pad8(sm.cnt[r]);
@@ -163,7 +174,7 @@ __device__ __forceinline__ bool issue_chunk(Prod& p, const SegSmem& sm, const __
   if (lane == 0) {
     const uint32_t bytes = (uint32_t)(rows * tl * 2);           // rows j0.. of the tile: contiguous
     mbar_arrive_expect_tx(bar, bytes);
-    if (fence) fence_proxy_async_smem();  // the generic reads above precede the async write
+    fence_proxy_async_smem();  // the generic reads above precede the async write
     bulk_g2s_hint(stage_addr, (p.phase ? cV : cK) + sm.base[r] + t0 * r + (long long)j0 * tl, bytes, bar,
                   policy);
   }
@@ -174,7 +185,7 @@ __device__ __forceinline__ bool issue_chunk(Prod& p, const SegSmem& sm, const __
     if (++p.phase == 2) {
       p.phase = 0;
       p.k += NW;
-      if (p.k < total) p.item = item_at(sm, p.k);
+      if (p.k < total) p.item = next_rr(sm, p.item, p.k);
     }
   }
   return true;
@@ -286,45 +297,24 @@ __device__ __forceinline__ void seg_cta_range(const long long* cuts, long long T
 constexpr int kMaxCtas = 1024;   // grid size bound (64-bit cost-line arithmetic)
 static_assert(kMaxCtas < (1 << 16), "udiv_small divides by the grid size");
 
-// Completion word of one (sequence, KV head) segment: bits 63..32 hold the epoch of the call that
-// arrived last, bits 31..16 the number of CTAs that call expects on the segment, bits 15..0 how many
-// have arrived. A word is clean when it is zero (never used) or holds a finished count. The first
-// CTA of a call replaces a clean word by (epoch, n, 1), the others count up, and the one that
-// completes the count merges the segment. Any other word (another epoch still counting, a count or
-// an expected value out of range) means an earlier call never finished or two calls overlap on
-// this workspace: the arrival raises VARRATE_ERR_CORRUPT and re-arms the word for its own call, so
-// the next call finds it clean. A replay of a captured launch keeps its epoch and finds its own
-// finished word, which is clean. Returns true for the CTA that completes the count.
-// The CTA that completes the count (it merges the segment next) takes one atomic: it first tries
-// (epoch, n, n - 1) -> (epoch, n, n); a lone CTA (n = 1) swaps its finished word in directly.
-__device__ __forceinline__ bool word_clean(unsigned long long w) {
-  const uint32_t on = (uint32_t)(w >> 16) & 0xFFFFu, oc = (uint32_t)w & 0xFFFFu;
-  return w == 0ull || (on >= 1u && on <= (uint32_t)kMaxCtas && oc == on);
-}
-__device__ bool seg_arrive(unsigned long long* word, uint32_t epoch, uint32_t n, int32_t* dev_status) {
-  const unsigned long long tag = ((unsigned long long)epoch << 32) | ((unsigned long long)n << 16);
-  if (n == 1) {
-    if (!word_clean(atomicExch(word, tag | 1ull))) raise_status(dev_status, VARRATE_ERR_CORRUPT);
-    return true;
-  }
-  unsigned long long old = atomicCAS(word, tag | (n - 1), tag | n);
-  if (old == (tag | (n - 1))) return true;
-  for (int tries = 0; tries < (1 << 16); ++tries) {   // one retry per concurrent arrival
-    const uint32_t oe = (uint32_t)(old >> 32), on = (uint32_t)(old >> 16) & 0xFFFFu;
-    const uint32_t oc = (uint32_t)old & 0xFFFFu;
-    const bool counting = oe == epoch && oc < on;
-    const bool bad = counting ? on != n : !word_clean(old);
-    const unsigned long long nw = (counting && !bad) ? old + 1ull : (tag | 1ull);
-    const unsigned long long prev = atomicCAS(word, old, nw);
-    if (prev == old) {
-      if (bad) raise_status(dev_status, VARRATE_ERR_CORRUPT);
-      return (uint32_t)(nw & 0xFFFFull) == n;
-    }
-    old = prev;
-  }
-  raise_status(dev_status, VARRATE_ERR_TIMEOUT);
-  return false;
-}
+// Completion counting (the first kDecodeCounterBytes of the workspace, DecodeHeader): a count of
+// the fused calls made on the workspace, and two sets of per-(sequence, KV head) arrival counters
+// with a grid-exit counter each. A call reads the call count once (after griddepcontrol.wait, so
+// the previous call has finished) and counts on the set of its parity with plain atomicAdd; it
+// never resets that set, and instead zeroes the other set, which the previous call used and the
+// next call will use. So every call starts from zero counters; counts left by an earlier call that
+// overlapped this one or gave up show as an arrival past the expected number (exactly detected:
+// VARRATE_ERR_CORRUPT), and are gone one call later without any action by the caller. The CTA that
+// brings the grid-exit counter to a multiple of the grid size advances the call count; replaying
+// a captured launch advances it the same way.
+struct DecodeHeader {
+  unsigned long long calls;         // fused calls completed on this workspace
+  uint32_t exits[2];                // CTAs that left the kernel, per parity
+  uint32_t pad[60];
+  uint32_t arrived[2][kDecodeMaxSegs];   // CTAs that finished segment seg, per parity
+};
+static_assert(sizeof(DecodeHeader) == kDecodeCounterBytes, "decode header layout");
+static_assert(offsetof(DecodeHeader, arrived) == 256, "counter sets start 256 bytes in");
 
 constexpr int kMaxTailFused = 256;   // exact tail tokens the fused kernel stages in the ring
 
@@ -513,14 +503,13 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
                   const __nv_bfloat16* __restrict__ basis_v, const __nv_bfloat16* __restrict__ qin,
                   const __nv_bfloat16* __restrict__ tail_k, const __nv_bfloat16* __restrict__ tail_v,
                   int n_tail, __nv_bfloat16* __restrict__ out, float* __restrict__ part,
-                  unsigned long long* __restrict__ seg_done, int32_t* __restrict__ dev_status, Shape s,
-                  int layer, uint32_t epoch) {
+                  DecodeHeader* __restrict__ hdr, int32_t* __restrict__ dev_status, Shape s,
+                  int layer) {
   extern __shared__ __align__(128) unsigned char smem[];
   unsigned char* ring = smem;                                     // NW * ST * STAGE
   static_assert((NW * ST * STAGE) % 16 == 0, "SegSmem must start 16-byte aligned");
   SegSmem& sm = *reinterpret_cast<SegSmem*>(smem + NW * ST * STAGE);
-  // the merge and combine buffers alias the ring; the ring is zeroed again after every merge so
-  // that it only ever holds finite coefficients or zeros
+  // the merge and combine buffers alias the ring (idle while a segment is merged)
   static_assert(sizeof(Merge) <= (size_t)NW * ST * STAGE, "merge buffers fit in the ring");
   Merge& mg = *reinterpret_cast<Merge*>(smem);
   __shared__ long long segW[64];                                  // per-sequence stream length
@@ -528,6 +517,7 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
   __shared__ long long cuts[kMaxCtas + 1];                        // start of CTA c's range
   __shared__ int n_empty;                                         // sequences with no coded tokens
   __shared__ int last_cta;                                        // this CTA closes the segment
+  __shared__ uint32_t parity;                                     // counter set of this call
   __shared__ uint64_t bar_all[NW * ST];                           // one full-barrier per ring stage
   __shared__ uint64_t bar_comb;                                   // U_V copy of a combine
 
@@ -540,20 +530,24 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
   // and waits (griddepcontrol.wait) for this grid to finish before it reads anything
   pdl_trigger();
   // self-contained setup first (it may overlap the tail of the preceding grid)
-  // the ring only ever holds finite coefficients or zeros
-  for (int i = tid; i < NW * ST * STAGE / 16; i += blockDim.x)
-    reinterpret_cast<uint4*>(ring)[i] = make_uint4(0, 0, 0, 0);
   if (tid < NW * ST) mbar_init(&bar_all[tid], 1);
   if (tid == NW * ST) mbar_init(&bar_comb, 1);
   fence_mbar_init();
   fence_proxy_async_smem();
   pdl_wait();   // everything below reads data written by earlier grids
+  if (tid == 0) parity = (uint32_t)(*reinterpret_cast<volatile unsigned long long*>(&hdr->calls) & 1ull);
   // stream length of every sequence of this layer (same for every head); poisoned tables -> 0
   for (int b = tid; b < s.B; b += blockDim.x) {
     const long long w = bucket_base[((long long)b * s.L + layer) * (kMaxR + 2) + kMaxR + 1];
     segW[b] = (w >= 0 && w <= s.cap) ? w : 0;
   }
   __syncthreads();
+  {   // the other set: used by the previous call (finished), counted on by the next one
+    uint32_t* other = hdr->arrived[parity ^ 1u];
+    for (int i = cta * (int)blockDim.x + tid; i < kDecodeMaxSegs; i += C * (int)blockDim.x) other[i] = 0u;
+    if (cta == 0 && tid == 0) hdr->exits[parity ^ 1u] = 0u;
+  }
+  uint32_t* arrived = hdr->arrived[parity];
   uint32_t n_issued = 0;   // chunks this warp has consumed (== index of its next chunk)
   int n_pending = 0;       // chunks issued but not yet consumed
   bool timed_out = false;  // this thread saw a bounded wait give up
@@ -674,10 +668,9 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
       int cons_k = pr.k;
       Item cons = pr.item;
 #pragma unroll
-      for (int i = 0; i < ST - 1; ++i)
-        // the ring was zeroed and fenced before the segment began: no fence for these
+      for (int i = 0; i < ST; ++i)   // every stage of the ring in flight
         if (issue_chunk(pr, sm, cK, cV, ring_w + ((n_issued + i) % ST) * STAGE,
-                        &bars[(n_issued + i) % ST], total, lane, policy, false)) ++n_pending;
+                        &bars[(n_issued + i) % ST], total, lane, policy)) ++n_pending;
       int c0, c1;   // the CTAs that share this segment (their partials are merged by the last one)
       seg_cta_range(cuts, T, C, P, W, c0, c1);
       __syncwarp();
@@ -694,11 +687,12 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
         return true;
       };
       auto next_chunk = [&]() {
-        // the consumed stage is free again: refill it with the chunk ST-1 ahead
+        // the consumed stage is free again: refill it with the chunk ST ahead, so that all the
+        // other stages stay in flight while the warp computes
         ++n_issued;
         --n_pending;
-        if (issue_chunk(pr, sm, cK, cV, ring_w + ((n_issued + ST - 2) % ST) * STAGE,
-                        &bars[(n_issued + ST - 2) % ST], total, lane, policy)) ++n_pending;
+        if (issue_chunk(pr, sm, cK, cV, ring_w + ((n_issued + ST - 1) % ST) * STAGE,
+                        &bars[(n_issued + ST - 1) % ST], total, lane, policy)) ++n_pending;
       };
 
       while (cons_k < total && !timed_out) {
@@ -724,22 +718,34 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
           const int j0 = jc << lgc, j1 = min(r, j0 + (1 << lgc));
 #pragma unroll 2
           for (int j16 = j0; j16 < j1; j16 += 16) {
-            uint4 qf = *reinterpret_cast<const uint4*>(&sm.qfrag[j16 >> 4][lane][0]);
-            if (j16 + 16 > r) {                          // warp-uniform: rows >= r in this k-step
-              const int jb = j16 + 2 * c;
-              qf.x = keep_rows(qf.x, jb, r); qf.z = keep_rows(qf.z, jb, r);
-              qf.y = keep_rows(qf.y, jb + 8, r); qf.w = keep_rows(qf.w, jb + 8, r);
-            }
+            const uint4 qf = *reinterpret_cast<const uint4*>(&sm.qfrag[j16 >> 4][lane][0]);
             // this lane's row of the 8x8 matrices: coefficient j, staged at row (j - chunk start)
             const int jrow = (j16 - j0) + (m >> 1) * 8 + r8;
             const int j = j0 + jrow;
             const uint32_t row_addr = st_addr + jrow * row_bytes;
             uint32_t a[ISL / 16][4];
-            int pg = full_tile ? (((m & 1) + j) & 15) : (((m & 1) + j) % ng);   // slot group 2 mt + (m & 1)
+            // stored position of slot group 2 mt + (m & 1) in row j: (group + j) mod ng; for a full
+            // tile every offset is computed on its own (no chain through the previous one)
+            uint32_t off[ISL / 16];
+            if (full_tile) {
+              const uint32_t o0 = (uint32_t)(((m & 1) + j) & 15) << 4;
 #pragma unroll
-            for (int mt = 0; mt < ISL / 16; ++mt) {
-              ldsm_x4_trans(row_addr + 16 * pg, a[mt]);
-              pg = wrap2(pg, ng);
+              for (int mt = 0; mt < ISL / 16; ++mt) off[mt] = (o0 + 32u * mt) & 255u;
+            } else {
+              int pg = ((m & 1) + j) % ng;
+#pragma unroll
+              for (int mt = 0; mt < ISL / 16; ++mt) { off[mt] = 16u * pg; pg = wrap2(pg, ng); }
+            }
+#pragma unroll
+            for (int mt = 0; mt < ISL / 16; ++mt) ldsm_x4_trans(row_addr + off[mt], a[mt]);
+            if (j16 + 16 > r) {   // warp-uniform: rows >= r of this k-step are not coefficients
+              // A fragment registers 0, 1 hold rows j16 + 2c (+1), registers 2, 3 rows 8 later
+              const int jb = j16 + 2 * c;
+              const uint32_t m0 = keep_rows(0xFFFFFFFFu, jb, r), m1 = keep_rows(0xFFFFFFFFu, jb + 8, r);
+#pragma unroll
+              for (int mt = 0; mt < ISL / 16; ++mt) {
+                a[mt][0] &= m0; a[mt][1] &= m0; a[mt][2] &= m1; a[mt][3] &= m1;
+              }
             }
 #pragma unroll
             for (int mt = 0; mt < ISL / 16; ++mt) mma_bf16_16816(sc[mt], a[mt], qf.x, qf.y);
@@ -823,14 +829,22 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
             const uint32_t row_addr = st_addr + jrow * row_bytes;
             const bool keep0 = jt * 16 + g8 < r, keep1 = jt * 16 + g8 + 8 < r;
             float t1[4] = {0.f, 0.f, 0.f, 0.f};
-            int pg = full_tile ? (((m >> 1) + j) & 15) : (((m >> 1) + j) % ng);  // slot group 2 kt + (m >> 1)
+            // stored position of slot group 2 kt + (m >> 1) (kt = 0..7) in row j, as in the K loop
+            uint32_t off[ISL / 16];
+            if (full_tile) {
+              const uint32_t o0 = (uint32_t)(((m >> 1) + j) & 15) << 4;
+#pragma unroll
+              for (int kt = 0; kt < ISL / 16; ++kt) off[kt] = (o0 + 32u * kt) & 255u;
+            } else {
+              int pg = ((m >> 1) + j) % ng;
+#pragma unroll
+              for (int kt = 0; kt < ISL / 16; ++kt) { off[kt] = 16u * pg; pg = wrap2(pg, ng); }
+            }
 #pragma unroll
             for (int kt = 0; kt < ISL / 16; kt += 2) {
               uint32_t a[4], b[4];
-              ldsm_x4(row_addr + 16 * pg, a);
-              pg = wrap2(pg, ng);
-              ldsm_x4(row_addr + 16 * pg, b);
-              pg = wrap2(pg, ng);
+              ldsm_x4(row_addr + off[kt], a);
+              ldsm_x4(row_addr + off[kt + 1], b);
               if (jt * 16 + 16 > r) {                    // warp-uniform: rows >= r in this tile
                 if (!keep0) { a[0] = a[2] = 0u; b[0] = b[2] = 0u; }
                 if (!keep1) { a[1] = a[3] = 0u; b[1] = b[3] = 0u; }
@@ -844,7 +858,7 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
           if (ok) { __syncwarp(); next_chunk(); }         // the last chunk of the item
         }
         cons_k += NW;
-        if (cons_k < total) cons = item_at(sm, cons_k);
+        if (cons_k < total) cons = next_rr(sm, cons, cons_k);
       }
       // drain: never leave bulk copies in flight into this ring (a copy whose wait gave up stays
       // counted in n_pending and is waited for once more before the CTA exits)
@@ -912,9 +926,12 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
       // the last CTA to finish this segment merges every partial of it
       __syncthreads();
       if (tid == 0) {
-        __threadfence();
-        last_cta = seg_arrive(&seg_done[seg], epoch, (uint32_t)(c1 - c0 + 1), dev_status);
-        if (last_cta) __threadfence();   // the other CTAs' partials (published before they arrived) are read next
+        // release: this CTA's partial (ordered before by the barrier) is visible to whoever sees
+        // the count; acquire: the last arrival then sees every other CTA's partial
+        const uint32_t n = (uint32_t)(c1 - c0 + 1);   // CTAs that share this segment
+        const uint32_t done = atom_add_acq_rel_gpu(&arrived[seg], 1u);
+        last_cta = done == n - 1u;
+        if (done >= n) raise_status(dev_status, VARRATE_ERR_CORRUPT);   // counts left by an earlier call
       }
       __syncthreads();
       if (last_cta && !dead) {
@@ -935,9 +952,7 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
     while (b < s.B && segW[b] == 0) ++b;
     more = b < s.B && seg_start(b, g) < hi_g;
     if (more && !dead) {
-      for (int i = tid; i < NW * ST * STAGE / 16; i += blockDim.x)
-        reinterpret_cast<uint4*>(ring)[i] = make_uint4(0, 0, 0, 0);
-      fence_proxy_async_smem();
+      fence_proxy_async_smem();   // the merge and combine wrote the ring: before the next copies
       __syncthreads();
     }
   }
@@ -966,6 +981,11 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
     if (n_comb > 0 && tid == 0) mbar_wait_bounded(&bar_comb, (n_comb - 1) & 1u, kWaitTries);
   }
   if (timed_out && lane == 0) raise_status(dev_status, VARRATE_ERR_TIMEOUT);
+  // the CTA that completes a multiple of the grid size of exits advances the call count (a
+  // multiple rather than exactly C - 1: the count then stays consistent whatever the set held)
+  __syncthreads();
+  if (tid == 0 && (atomicAdd(&hdr->exits[parity], 1u) + 1u) % (uint32_t)C == 0u)
+    atomicAdd(&hdr->calls, 1ull);
 }
 
 }  // namespace
@@ -989,10 +1009,18 @@ bool decode_mma_supported(const Shape& s, int n_tail, int num_sms) {
 int launch_decode_mma(const Shape& s, const varrate_packed& c, const void* basis_k,
                       const void* basis_v, const void* q, int layer, const void* tail_k,
                       const void* tail_v, int n_tail, void* out, int32_t* dev_status,
-                      unsigned long long* seg_done, float* part, uint32_t epoch, int num_sms,
-                      cudaStream_t st) {
+                      void* header, float* part, int num_sms, cudaStream_t st) {
   const size_t smem = decode_mma_smem_bytes();
-  cudaFuncSetAttribute(decode_mma_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  // the shared-memory opt-in is a per-device property of the function: set once per device
+  static std::atomic<int> smem_set[64];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64 ||
+      smem_set[dev].load(std::memory_order_acquire) == 0) {
+    if (cudaFuncSetAttribute(decode_mma_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
+        cudaSuccess)
+      return -1;
+    if (dev >= 0 && dev < 64) smem_set[dev].store(1, std::memory_order_release);
+  }
   // the grid may be scheduled while its predecessor drains (programmatic dependent launch); it
   // waits on griddepcontrol.wait before touching anything an earlier operation wrote
   cudaLaunchAttribute pdl[1];
@@ -1009,7 +1037,7 @@ int launch_decode_mma(const Shape& s, const varrate_packed& c, const void* basis
                      (const int64_t*)c.bucket_base, (const __nv_bfloat16*)basis_k,
                      (const __nv_bfloat16*)basis_v, (const __nv_bfloat16*)q,
                      (const __nv_bfloat16*)tail_k, (const __nv_bfloat16*)tail_v, n_tail,
-                     (__nv_bfloat16*)out, part, seg_done, dev_status, s, layer, epoch);
+                     (__nv_bfloat16*)out, part, reinterpret_cast<DecodeHeader*>(header), dev_status, s, layer);
   return 1;
 }
 

@@ -15,10 +15,11 @@ namespace {
 
 // Scratch for every call of this entry point on a device. Every GPU that loads the library holds
 // it until the process exits. Calls share it and it keeps the previous call's contents. It starts
-// zero-filled (as a __device__ array without initialiser is); its first part holds the decode
-// kernel's completion words, which each call leaves in a finished state (or re-arms, raising
-// VARRATE_ERR_CORRUPT once, if an earlier call overlapped it or gave up), and the decode kernels
-// write every other element they later read, so nothing has to be cleared between calls.
+// zero-filled (as a __device__ array without initialiser is); its first part is the decode
+// kernel's header (a call count and two alternating sets of arrival counters, each call clearing
+// the set the next call uses, so counts left by an overlapping or timed-out call are reported once
+// as VARRATE_ERR_CORRUPT and gone one call later), and the decode kernels write every other
+// element they later read, so nothing has to be cleared between calls.
 constexpr size_t kScratchBytes = size_t(4) << 20;   // 4 MiB
 static __device__ __align__(256) unsigned char g_decode_scratch[kScratchBytes];
 

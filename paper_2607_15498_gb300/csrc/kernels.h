@@ -48,11 +48,11 @@ int launch_project_tc(const Shape& s, const void* k, const void* v, const void* 
                       int num_sms, cudaStream_t st);
 
 // ---- step 4: decode attention
-// The decode workspace starts with a fixed block of per-(sequence, KV head) completion words (64
-// bits each, used by the bf16 tensor-core kernel: epoch of the last call, CTAs it expected, CTAs
-// arrived); the rest of the workspace is scratch that every call writes before it reads.
+// The decode workspace starts with a fixed header used by the bf16 tensor-core kernel: a count of
+// its calls and two alternating sets of per-(sequence, KV head) arrival counters (decode_mma.cu);
+// the rest of the workspace is scratch that every call writes before it reads.
 constexpr int kDecodeMaxSegs = 4096;
-constexpr size_t kDecodeCounterBytes = (size_t)kDecodeMaxSegs * sizeof(unsigned long long);
+constexpr size_t kDecodeCounterBytes = 256 + 2 * (size_t)kDecodeMaxSegs * sizeof(uint32_t);
 int decode_splits(const Shape& s, int num_sms);
 size_t decode_ws_bytes(const Shape& s, int num_sms);
 // bf16 tensor-core decode (decode_mma.cu)
@@ -62,12 +62,10 @@ bool decode_mma_supported(const Shape& s, int n_tail, int num_sms);
 int launch_decode_mma(const Shape& s, const varrate_packed& c, const void* basis_k,
                       const void* basis_v, const void* q, int layer, const void* tail_k,
                       const void* tail_v, int n_tail, void* out, int32_t* dev_status,
-                      unsigned long long* seg_done, float* part, uint32_t epoch, int num_sms,
-                      cudaStream_t st);
-// `epoch` tags the call in the completion words (nonzero; a new value for every call).
+                      void* header, float* part, int num_sms, cudaStream_t st);
 int launch_decode(const Shape& s, const varrate_packed& cache, const void* basis_k,
                   const void* basis_v, const void* q, int layer, const void* tail_k,
                   const void* tail_v, int n_tail, void* out, int32_t* dev_status, void* ws,
-                  uint32_t epoch, int num_sms, cudaStream_t st);
+                  int num_sms, cudaStream_t st);
 
 }  // namespace vr
