@@ -503,6 +503,76 @@ def sweep_reuse(V, wl, dev, peak, stream, n_batches, n_window, n_decode):
             "l2": "packed cache of all layers (3.4 GB) read per step (> L2)"}
 
 
+def sweep_quant(V, wl, dev, peak, stream, decode_steps, bits_list=(4, 8)):
+    """Quantized coefficients on a llama32-shaped stack: quantize time per encode, and decode on the
+    quantized cache (the general kernels) with its algorithmic bytes (codes and group parameters of
+    K and V, bases, queries and outputs), next to the bf16 cache's footprint."""
+    cfg = V.make_config(wl.n_layers, wl.n_kv_heads, wl.group, wl.n_ctx, batch=wl.batch,
+                        budget_frac=wl.budget_frac, r_min=wl.r_min, window=wl.window, dtype=V.BF16)
+    k, v, qw, bk, bv = synth.stack_inputs(wl, device=dev)
+    packed = V.PackedCache.allocate(cfg, dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    V.check(V.varrate_encode(cfg, qw, k, v, bk, bv, None, packed, None, status,
+                             V.workspace(cfg, V.CALL_ENCODE, dev), stream), "varrate_encode")
+    torch.cuda.synchronize()
+    del k, v, qw
+    d = wl.head_dim
+    fixed = 2 * wl.n_kv_heads * d * d * 2 + 2 * wl.batch * wl.n_q_heads * d * 2
+    bf16_bytes = sum(coded_bytes_per_layer(packed, cfg))
+    qdec = torch.stack([synth.stack_decode_queries(wl, l, decode_steps, device=dev)
+                        for l in range(wl.n_layers)], dim=1)
+    out = torch.empty((wl.batch, wl.n_q_heads, d), dtype=torch.bfloat16, device=dev)
+    ws = V.workspace(cfg, V.CALL_DECODE, dev)
+    res = {}
+    for bits in bits_list:
+        qp = V.QPackedCache.allocate(cfg, packed, bits, dev)
+        times = []
+        for i in range(4):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            V.check(V.varrate_quantize(cfg, packed, qp, status, stream), "varrate_quantize")
+            e1.record(stream)
+            torch.cuda.synchronize()
+            if i:
+                times.append(e0.elapsed_time(e1))
+        q_bytes = int(qp.qbase[:, :, -1].sum().item()) * wl.n_kv_heads * 2   # all layers
+
+        def phase(n):
+            for s_ in range(n):
+                for l in range(wl.n_layers):
+                    V.check(V.varrate_decode_attn_q(cfg, qp, bk, bv, qdec[s_, l], l, None, None, 0,
+                                                    out, status, ws, None), "varrate_decode_attn_q")
+        phase(1)
+        g = capture(lambda: phase(decode_steps))
+        g.replay()
+        torch.cuda.synchronize()
+        dts = []
+        for _ in range(3):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            g.replay()
+            e1.record(stream)
+            torch.cuda.synchronize()
+            dts.append(e0.elapsed_time(e1))
+        dec_ms = statistics.median(dts)
+        n_calls = decode_steps * wl.n_layers
+        step_bytes = q_bytes + wl.n_layers * fixed
+        gbs = decode_steps * step_bytes / (dec_ms * 1e-3) / 1e9
+        res[f"{bits}bit"] = {
+            "quantize_ms_per_layer": round(statistics.median(times) / wl.n_layers, 4),
+            "footprint_vs_bf16": round(q_bytes / bf16_bytes, 4),
+            "decode_us_per_layer_call": round(dec_ms * 1e3 / n_calls, 2),
+            "decode_bytes_per_layer_call": int(step_bytes / wl.n_layers),
+            "decode_gbs": round(gbs, 1), "decode_frac_of_hbm_peak": round(gbs / peak, 4),
+            "decode_status": V.status_string(int(status.item())),
+            "decode_kernels": "general split-and-combine kernels (CUDA cores), graph-replayed"}
+        del g, qp
+    res["workload"] = workload_desc(wl)
+    del packed, qdec
+    torch.cuda.empty_cache()
+    return res
+
+
 def run_sweep(args, peak):
     """The other seeded configurations, each with its own encode and decode numbers."""
     from paper_2607_15498_gb300 import varrate as V
@@ -520,6 +590,8 @@ def run_sweep(args, peak):
     wl = synth.workload("reuse")
     out["reuse"] = sweep_reuse(V, wl, dev, peak, stream, n_batches=args.reuse_batches,
                                n_window=32, n_decode=wl.decode_steps)
+    out["llama32_quantized"] = sweep_quant(V, synth.workload("llama32", n_layers=4), dev, peak,
+                                           stream, decode_steps=32)
     return out
 
 

@@ -106,6 +106,27 @@ typedef struct {
   int64_t cap_elems;      /* elements per stream, >= varrate_packed_cap_elems() */
 } varrate_packed;
 
+/* Quantized packed cache: the coefficients of a varrate_packed cache in group-wise b-bit form
+ * (Sec. 3.3, "Composability"; the allocation and bucket tables are unchanged). A group is 32
+ * consecutive slots of one coefficient row of a 128-slot tile (one coefficient of up to 32 tokens of
+ * equal rank, in bucket order, bucket padding slots included as zeros); its values x map to codes
+ *   lo = fp16(min x), step = fp16(min(fl32(max x - lo) / (2^b - 1), 65504)),
+ *   code = clip(rint(fl32(fl32(x - lo) / step)), 0, 2^b - 1)   (step == 0: code 0),
+ * and back to x^ = fl32(lo + fl32(code * step)). Stream (b, l, g, kv) occupies qcap_bytes bytes from
+ * data + (((b * L + l) * G + g) * 2 + kv) * qcap_bytes; bucket r starts at byte qbase[b][l][r]; its
+ * tiles follow back to back (the last one pad8(n_r) mod 128 slots), each r rows of
+ * qrow(tl) = roundup16(tl * b / 8 + 4 * ceil(tl / 32)) bytes: row j of tile i at
+ * qbase[r] + i * r * qrow(128) + j * qrow(tl) holds the codes of slots 0 .. tl - 1 (b = 4: two per
+ * byte, the even slot in the low nibble; b = 8: one per byte), then (fp16 lo, fp16 step) of each
+ * group of 32 slots, then zeros. Slot p of the tile is bucket position 128 i + p. */
+typedef struct {
+  uint8_t* data;                /* [B][L][G][2][qcap_bytes] */
+  int64_t* qbase;               /* [B][L][d + 2] byte offset of bucket r in a stream */
+  const int32_t* bucket_count;  /* [B][L][d + 1] the source cache's bucket counts */
+  int32_t bits;                 /* 4 or 8 */
+  int64_t qcap_bytes;           /* bytes per stream, >= varrate_qpacked_cap_bytes(cfg, bits) */
+} varrate_qpacked;
+
 /* Which call a workspace is sized for. */
 typedef enum {
   VARRATE_CALL_SALIENCE = 0,
@@ -206,6 +227,30 @@ varrate_status varrate_decode_attn(const varrate_config* cfg, const varrate_pack
                                    int32_t layer, const void* tail_k, const void* tail_v,
                                    int32_t n_tail, void* out, int32_t* dev_status, void* ws,
                                    size_t ws_bytes, void* stream);
+
+/* Upper bound on the bytes of one quantized stream for any allocation within the budget:
+ * with S = max(B_c, r_min * (N - w)) + w * d, R = sum_{r = r_min..d} r and F = qrow(128):
+ * roundup16(ceil(F * (S + 7 R) / 128) + 19 R). Returns -1 if cfg or bits is invalid. */
+int64_t varrate_qpacked_cap_bytes(const varrate_config* cfg, int32_t bits);
+
+/* Quantize a bf16 packed cache (every stream of every (sequence, layer)) into `out` (layout above):
+ * fills out->qbase from in->bucket_count and writes the codes and group parameters. out->bits is 4
+ * or 8 and out->bucket_count must be in->bucket_count. A table that does not fit in->cap_elems or
+ * out->qcap_bytes raises VARRATE_ERR_CORRUPT in *dev_status and leaves that (b, l) unwritten.
+ * dtype must be VARRATE_BF16 (VARRATE_ERR_UNSUPPORTED otherwise). No workspace. */
+varrate_status varrate_quantize(const varrate_config* cfg, const varrate_packed* in,
+                                varrate_qpacked* out, int32_t* dev_status, void* stream);
+
+/* Decode attention of one layer on a quantized cache: the same mathematics and arguments as
+ * varrate_decode_attn with each stored coefficient c replaced by its dequantized value x^ (fp32),
+ * computed by the general kernels (query rotation, split over tokens, combine); ws as for
+ * varrate_decode_attn (varrate_workspace_bytes(cfg, VARRATE_CALL_DECODE)); 0 <= n_tail <= 4096;
+ * dtype VARRATE_BF16 only (queries, bases, tail and output bf16). */
+varrate_status varrate_decode_attn_q(const varrate_config* cfg, const varrate_qpacked* cache,
+                                     const void* basis_k, const void* basis_v, const void* q,
+                                     int32_t layer, const void* tail_k, const void* tail_v,
+                                     int32_t n_tail, void* out, int32_t* dev_status, void* ws,
+                                     size_t ws_bytes, void* stream);
 
 /* Decode attention without caller workspace (the paper has no counterpart: this is an interface
  * for callers that cannot allocate device memory, such as a plugin that a host framework hands only

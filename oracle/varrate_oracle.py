@@ -399,3 +399,105 @@ def encode_layer(q_win, k, v, basis_k, basis_v, group, budget_frac, r_min, pool_
     cv = np.stack([project(v[g], basis_v[g]) for g in range(G)])
     return dict(sal=sal32, ranks=ranks, status=status, total=total, count=count, base=base,
                 pos=pos, perm=perm, coef_k=ck, coef_v=cv)
+
+
+# ------------------------------------------- coefficient quantization (Sec. 3.3, "Composability")
+
+# The paper states that the coefficients c_t can be quantized with standard group-wise b-bit
+# quantization without touching the allocation. Reading taken here: a group is 32 consecutive slots
+# (tokens of one rank, in bucket order) of one coefficient row j inside a 128-slot tile of the
+# packed layout, so a group holds one coefficient of up to 32 tokens of equal rank; quantization is
+# asymmetric min-max with the group's offset and step stored in fp16:
+#     lo = fp16(min), step = fp16(fl32(max - lo) / (2^b - 1)),
+#     code = clip(rint(fl32(fl32(x - lo) / step)), 0, 2^b - 1)   (step = 0: code 0),
+#     x^ = fl32(lo + fl32(code * step)).
+# Padding slots of a bucket (zeros) belong to the group of their tile like the others.
+
+QGROUP = 32
+
+
+def qrow_bytes(tl: int, bits: int) -> int:
+    """Bytes of one quantized coefficient row of a tile of tl slots: the codes (tl * bits / 8),
+    then (fp16 offset, fp16 step) per group of 32 slots, rounded up to 16 bytes."""
+    raw = tl * bits // 8 + 4 * ((tl + QGROUP - 1) // QGROUP)
+    return (raw + 15) // 16 * 16
+
+
+def quantize_group(x, bits: int):
+    """One group: float32 values -> (uint8 codes, fp16 offset, fp16 step)."""
+    x = np.asarray(x, dtype=np.float32)
+    qmax = np.float32(2 ** bits - 1)
+    lo = np.float16(x.min())
+    lo32 = np.float32(lo)
+    # a range beyond the fp16 range saturates the step at the largest finite fp16
+    step = np.float16(min(np.float32(np.float32(x.max()) - lo32) / qmax, np.float32(65504.0)))
+    s32 = np.float32(step)
+    if s32 == 0:
+        return np.zeros(x.size, dtype=np.uint8), lo, step
+    with np.errstate(over="ignore", invalid="ignore"):
+        q = np.rint(((x - lo32).astype(np.float32) / s32).astype(np.float32))
+    q = np.clip(q, 0, qmax)
+    return q.astype(np.uint8), lo, step
+
+
+def dequantize_group(codes, lo, step):
+    """x^ = fl32(lo + fl32(code * step)) (separately rounded multiply and add)."""
+    prod = (np.asarray(codes, dtype=np.float32) * np.float32(step)).astype(np.float32)
+    return (np.float32(lo) + prod).astype(np.float32)
+
+
+def qpack_tables(count, r_min: int, r_max: int, bits: int) -> np.ndarray:
+    """Byte offset of each rank bucket in a quantized stream (int64 [r_max + 2]): bucket r holds
+    its tiles (128 slots; the last one pad8(n_r) mod 128 slots) back to back, r rows each."""
+    qbase = np.zeros(r_max + 2, dtype=np.int64)
+    full = qrow_bytes(128, bits)
+    for r in range(r_min, r_max + 1):
+        n8 = (int(count[r]) + 7) // 8 * 8
+        last = n8 % 128
+        qbase[r + 1] = qbase[r] + r * ((n8 // 128) * full + (qrow_bytes(last, bits) if last else 0))
+    return qbase
+
+
+def qpacked_cap_bytes(n_ctx: int, head_dim: int, window: int, budget_frac: float, r_min: int,
+                      bits: int) -> int:
+    """Static upper bound on the bytes of one quantized stream for any allocation: with
+    S = max(B_c, r_min |C|) + w d rank units (+ 7 padding slots per bucket and row), a full-tile
+    row costs qrow_bytes(128) / 128 per unit and a short last tile at most 19 bytes per row more
+    than its share (group parameters of a partial group, 16-byte rounding)."""
+    n_coded = n_ctx - window
+    s = max(coded_budget(n_ctx, head_dim, window, budget_frac), r_min * n_coded, 0) \
+        + window * head_dim
+    rsum = sum(range(r_min, head_dim + 1))
+    full = qrow_bytes(128, bits)
+    cap = (full * (s + 7 * rsum) + 127) // 128 + 19 * rsum
+    return (cap + 15) // 16 * 16
+
+
+def quantize_coefficients(coef, ranks, count, pos, bits: int):
+    """Quantize one stream given its per-token coefficients coef [N][d] (float32: the stored values)
+    and the bucket tables. Returns (codes [N][d] uint8 (0 beyond each rank), lo [N][d] fp16 and
+    step [N][d] fp16 of the group each coefficient belongs to, dequantized [N][d] float32)."""
+    coef = np.asarray(coef, dtype=np.float32)
+    ranks = np.asarray(ranks, dtype=np.int64)
+    N, d = coef.shape
+    codes = np.zeros((N, d), dtype=np.uint8)
+    lo = np.zeros((N, d), dtype=np.float16)
+    step = np.zeros((N, d), dtype=np.float16)
+    deq = np.zeros((N, d), dtype=np.float32)
+    for r in np.unique(ranks):
+        toks = np.nonzero(ranks == r)[0]
+        order = toks[np.argsort(np.asarray(pos)[toks], kind="stable")]   # bucket order
+        n = order.size
+        n8 = (n + 7) // 8 * 8
+        for g0 in range(0, n8, QGROUP):                 # groups never cross a 128-slot tile
+            g1 = min(g0 + QGROUP, n8, (g0 // 128 + 1) * 128)
+            members = order[g0:min(g1, n)]
+            n_pad = (g1 - g0) - members.size            # padding slots of the bucket: zeros
+            for j in range(int(r)):
+                x = np.concatenate([coef[members, j], np.zeros(n_pad, dtype=np.float32)])
+                q, a, s = quantize_group(x, bits)
+                codes[members, j] = q[: members.size]
+                lo[members, j] = a
+                step[members, j] = s
+                deq[members, j] = dequantize_group(q[: members.size], a, s)
+    return codes, lo, step, deq

@@ -102,6 +102,25 @@ bool aligned16(std::initializer_list<const void*> ps) {
   return true;
 }
 
+int64_t qcap_bytes(const varrate_config* c, int bits) {
+  const int64_t n_coded = c->n_ctx - c->window;
+  int64_t sum = coded_budget(c);
+  if ((int64_t)c->r_min * n_coded > sum) sum = (int64_t)c->r_min * n_coded;
+  if (sum < 0) sum = 0;
+  sum += (int64_t)c->window * c->head_dim;
+  int64_t rsum = 0;
+  for (int r = c->r_min; r <= c->head_dim; ++r) rsum += r;
+  const int64_t full = vr::qrow_bytes(128, bits);
+  const int64_t cap = (full * (sum + 7 * rsum) + 127) / 128 + 19 * rsum;
+  return (cap + 15) & ~int64_t(15);
+}
+
+bool qpacked_ok(const varrate_config* c, const varrate_qpacked* p) {
+  return p && p->data && p->qbase && p->bucket_count && (p->bits == 4 || p->bits == 8) &&
+         p->qcap_bytes >= qcap_bytes(c, p->bits) && (p->qcap_bytes % 16) == 0 &&
+         aligned16({p->data, p->qbase, p->bucket_count});
+}
+
 bool packed_ok(const varrate_config* c, const varrate_packed* p) {
   return p && p->coef && p->bucket_count && p->bucket_base && p->perm && p->pos && p->ranks &&
          p->cap_elems >= cap_elems(c) && (p->cap_elems % 8) == 0 &&
@@ -232,6 +251,47 @@ varrate_status varrate_decode_attn(const varrate_config* cfg, const varrate_pack
   if (vr::launch_decode(s, *cache, basis_k, basis_v, q, layer, tail_k, tail_v, n_tail, out, dev_status,
                         ws, num_sms(), (cudaStream_t)stream) < 0)
     return VARRATE_ERR_CUDA;
+  return launched();
+}
+
+int64_t varrate_qpacked_cap_bytes(const varrate_config* cfg, int32_t bits) {
+  if (check(cfg) != VARRATE_OK || (bits != 4 && bits != 8)) return -1;
+  return qcap_bytes(cfg, bits);
+}
+
+varrate_status varrate_quantize(const varrate_config* cfg, const varrate_packed* in,
+                                varrate_qpacked* out, int32_t* dev_status, void* stream) {
+  varrate_status st = check(cfg);
+  if (st != VARRATE_OK) return st;
+  if (cfg->dtype != VARRATE_BF16) return VARRATE_ERR_UNSUPPORTED;
+  if (!packed_ok(cfg, in) || !qpacked_ok(cfg, out) || out->bucket_count != in->bucket_count)
+    return VARRATE_ERR_ARG;
+  if (!aligned16({dev_status})) return VARRATE_ERR_ARG;
+  const Shape s = make_shape(cfg, in->cap_elems);
+  if ((int64_t)s.B * s.L > 65535) return VARRATE_ERR_UNSUPPORTED;   // grid.y of the quantize kernel
+  vr::launch_quantize(s, *in, *out, dev_status, (cudaStream_t)stream);
+  return launched();
+}
+
+varrate_status varrate_decode_attn_q(const varrate_config* cfg, const varrate_qpacked* cache,
+                                     const void* basis_k, const void* basis_v, const void* q,
+                                     int32_t layer, const void* tail_k, const void* tail_v,
+                                     int32_t n_tail, void* out, int32_t* dev_status, void* ws,
+                                     size_t ws_bytes_, void* stream) {
+  varrate_status st = check(cfg);
+  if (st != VARRATE_OK) return st;
+  if (cfg->dtype != VARRATE_BF16) return VARRATE_ERR_UNSUPPORTED;
+  if (!qpacked_ok(cfg, cache) || !basis_k || !basis_v || !q || !out) return VARRATE_ERR_ARG;
+  if (layer < 0 || layer >= cfg->n_layers || n_tail < 0) return VARRATE_ERR_ARG;
+  if (n_tail > 4096) return VARRATE_ERR_UNSUPPORTED;
+  if (n_tail > 0 && (!tail_k || !tail_v)) return VARRATE_ERR_ARG;
+  if (!aligned16({basis_k, basis_v, q, tail_k, tail_v, out, dev_status, ws})) return VARRATE_ERR_ARG;
+  const size_t need = ws_bytes(cfg, VARRATE_CALL_DECODE);
+  if (ws_bytes_ < need || ws == nullptr) return VARRATE_ERR_WORKSPACE;
+  const Shape s = make_shape(cfg, cap_elems(cfg));
+  (void)dev_status;
+  vr::launch_decode_q(s, *cache, basis_k, basis_v, q, layer, tail_k, tail_v, n_tail, out, ws,
+                      num_sms(), (cudaStream_t)stream);
   return launched();
 }
 

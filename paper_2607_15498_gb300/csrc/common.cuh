@@ -2,6 +2,7 @@
 #pragma once
 
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -56,6 +57,14 @@ __device__ __forceinline__ void load8_stream(const float* p, float (&f)[8]) {
 }
 
 __device__ __forceinline__ int64_t pad8(int64_t n) { return (n + 7) & ~int64_t(7); }
+
+// Bytes of one quantized coefficient row of a tile of tl slots (tl a multiple of 8): the codes
+// (tl * bits / 8 bytes), then an (fp16 offset, fp16 step) pair per group of 32 slots, rounded up
+// to 16 bytes.
+__host__ __device__ __forceinline__ int qrow_bytes(int tl, int bits) {
+  const int raw = tl * bits / 8 + 4 * ((tl + 31) / 32);
+  return (raw + 15) & ~15;
+}
 
 // Read-only 16-byte global load issued exactly where it is written (volatile: the compiler may not
 // sink it past later barriers), so its latency overlaps with the work that follows.

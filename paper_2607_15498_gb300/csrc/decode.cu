@@ -50,6 +50,68 @@ template <> struct Frag<float> {
   }
 };
 
+// Quantized 8-slot row fragment (group-wise b-bit codes, varrate_qpacked layout): the raw codes of
+// slots p0 .. p0 + 7 of one coefficient row (one 32-slot group) and the group's (offset, step);
+// get(i) dequantizes slot p0 + i as fl32(lo + fl32(code * step)).
+template <int BITS> struct QFrag {
+  uint32_t w0, w1;
+  float lo, st;
+  __device__ __forceinline__ void zero() { w0 = w1 = 0u; lo = 0.f; st = 0.f; }
+  __device__ __forceinline__ void load(const uint8_t* row, int p0, int tl) {
+    if (BITS == 4) {
+      w0 = __ldcs(reinterpret_cast<const unsigned int*>(row + (p0 >> 1)));
+      w1 = 0u;
+    } else {
+      const uint2 u = __ldcs(reinterpret_cast<const uint2*>(row + p0));
+      w0 = u.x; w1 = u.y;
+    }
+    const __half2 par = *reinterpret_cast<const __half2*>(row + tl * BITS / 8 + 4 * (p0 >> 5));
+    lo = __low2float(par);
+    st = __high2float(par);
+  }
+  __device__ __forceinline__ float get(int i) const {
+    const uint32_t c = BITS == 4 ? (w0 >> (4 * i)) & 15u : ((i < 4 ? w0 : w1) >> (8 * (i & 3))) & 255u;
+    return __fadd_rn(lo, __fmul_rn((float)c, st));
+  }
+};
+
+// Where the split kernel reads coefficient rows from. DenseSrc: the packed cache of `T` elements
+// (bucket offsets from its table). QuantSrc: the quantized cache (bucket element offsets rebuilt
+// from the counts, byte offsets from qbase).
+template <typename T> struct DenseSrc {
+  using F = Frag<T>;
+  static constexpr bool kTableBase = true;
+  const T* coef;
+  const int64_t* bucket_base;
+  int64_t stride;   // elements per stream
+  const T* cK;
+  const T* cV;
+  __device__ __forceinline__ void bind(int64_t stream0) { cK = coef + stream0 * stride; cV = cK + stride; }
+  __device__ __forceinline__ void load(F& f, int kv, int r, long long b0, long long qb0, long long n8,
+                                       long long s0, int j) const {
+    (void)qb0;
+    f.load((kv ? cV : cK) + b0 + coef_offset(r, n8, s0, j));
+  }
+};
+template <int BITS> struct QuantSrc {
+  using F = QFrag<BITS>;
+  static constexpr bool kTableBase = false;
+  const uint8_t* data;
+  const int64_t* qbase;
+  int64_t stride;   // bytes per stream
+  const uint8_t* qK;
+  const uint8_t* qV;
+  __device__ __forceinline__ void bind(int64_t stream0) { qK = data + stream0 * stride; qV = qK + stride; }
+  __device__ __forceinline__ void load(F& f, int kv, int r, long long b0, long long qb0, long long n8,
+                                       long long s0, int j) const {
+    (void)b0;
+    const long long it = s0 >> 7;
+    const int p0 = (int)(s0 & 127);
+    const int tl = (int)min(128ll, n8 - (it << 7));
+    f.load((kv ? qV : qK) + qb0 + it * r * qrow_bytes(128, BITS) + (long long)j * qrow_bytes(tl, BITS), p0, tl);
+  }
+};
+
 // v[32] holds partials of 32 (head, row) pairs; afterwards v[0] of lane i is the warp-wide sum of
 // pair i (each halving step keeps the half selected by the lane's bit and trades the other).
 __device__ __forceinline__ float transpose_reduce32(float (&v)[32]) {
@@ -95,16 +157,16 @@ decode_rotate_kernel(const T* __restrict__ q, const T* __restrict__ basis_k, flo
   }
 }
 
-template <typename T, int GP>
+template <class Src, int GP>
 __global__ void __launch_bounds__(256, (GP == 4 || GP == 2) ? 2 : 1)
-decode_split_kernel(const T* __restrict__ coef, const int32_t* __restrict__ bucket_count,
-                    const int64_t* __restrict__ bucket_base, const float* __restrict__ qt,
-                    float* __restrict__ part, Shape s, int layer, int S) {
+decode_split_kernel(Src src, const int32_t* __restrict__ bucket_count, const float* __restrict__ qt,
+                    float* __restrict__ part, Shape s, int layer, int S, long long table_cap) {
   constexpr int RG = 32 / GP;             // value rows per transpose-reduction
   constexpr int NACC = kHeadDim / RG;     // output coordinates owned per lane
   __shared__ __align__(16) float q_s[kHeadDim][GP];
   __shared__ int cnt[kMaxR + 1];
   __shared__ long long base[kMaxR + 2];
+  __shared__ long long qb[kMaxR + 2];   // quantized source: byte offset of each bucket
   __shared__ float wM[kWarps][GP], wL[kWarps][GP];
   __shared__ float wacc[kWarps][GP][kHeadDim];
 
@@ -113,7 +175,19 @@ decode_split_kernel(const T* __restrict__ coef, const int32_t* __restrict__ buck
   const int64_t bl = (int64_t)b * s.L + layer;
   for (int r = tid; r <= kMaxR + 1; r += blockDim.x) {
     if (r <= kMaxR) cnt[r] = bucket_count[bl * (kMaxR + 1) + r];
-    base[r] = bucket_base[bl * (kMaxR + 2) + r];
+    if constexpr (Src::kTableBase) base[r] = src.bucket_base[bl * (kMaxR + 2) + r];
+    else qb[r] = src.qbase[bl * (kMaxR + 2) + r];
+  }
+  if constexpr (!Src::kTableBase) {   // element offsets of the buckets, as the packed table has them
+    __syncthreads();
+    if (tid == 0) {
+      long long acc = 0;
+      for (int r = 0; r <= kMaxR; ++r) {
+        base[r] = acc;
+        if (r >= s.r_min && r <= s.r_max) acc += (long long)r * pad8(cnt[r]);
+      }
+      base[kMaxR + 1] = acc;
+    }
   }
   for (int i = tid; i < kHeadDim * GP; i += blockDim.x) {
     const int j = i / GP, hh = i % GP;
@@ -128,10 +202,9 @@ decode_split_kernel(const T* __restrict__ coef, const int32_t* __restrict__ buck
   for (int a = 0; a < NACC; ++a) acc[a] = 0.f;
 
   const long long W = base[kMaxR + 1];
-  const bool table_ok = W <= s.cap;
+  const bool table_ok = W <= s.cap && (Src::kTableBase || qb[kMaxR + 1] <= table_cap);
   const long long lo = table_ok ? W * split / S : 0, hi = table_ok ? W * (split + 1) / S : 0;
-  const T* cK = coef + ((bl * s.G + g) * 2) * s.cap;
-  const T* cV = cK + s.cap;
+  src.bind((bl * s.G + g) * 2);
   int counter = 0;
   for (int r = s.r_min; r <= s.r_max && table_ok; ++r) {
     const int n = cnt[r];
@@ -145,8 +218,7 @@ decode_split_kernel(const T* __restrict__ coef, const int32_t* __restrict__ buck
       if ((counter % kWarps) != warp) continue;
       const long long s0 = it * kItem + lane * 8;
       const bool lane_ok = lane < kItem / 8 && s0 < n8;   // lanes 16..31 idle: 8 slots per lane
-      const T* kp = cK + b0;
-      const T* vp = cV + b0;
+      const long long qb0 = Src::kTableBase ? 0 : qb[r];
 
       // scores for 8 slots x GP heads
       float sc[GP][8];
@@ -155,10 +227,10 @@ decode_split_kernel(const T* __restrict__ coef, const int32_t* __restrict__ buck
 #pragma unroll
         for (int i = 0; i < 8; ++i) sc[h][i] = 0.f;
       for (int j0 = 0; j0 < r; j0 += 8) {
-        Frag<T> f[8];
+        typename Src::F f[8];
 #pragma unroll
         for (int jj = 0; jj < 8; ++jj) {
-          if (lane_ok && j0 + jj < r) f[jj].load(kp + coef_offset(r, n8, s0, j0 + jj));
+          if (lane_ok && j0 + jj < r) src.load(f[jj], 0, r, b0, qb0, n8, s0, j0 + jj);
           else f[jj].zero();
         }
 #pragma unroll
@@ -206,10 +278,10 @@ decode_split_kernel(const T* __restrict__ coef, const int32_t* __restrict__ buck
 #pragma unroll
       for (int gi = 0; gi < NACC; ++gi) {
         if (gi * RG >= r) break;
-        Frag<T> f[RG];
+        typename Src::F f[RG];
 #pragma unroll
         for (int jj = 0; jj < RG; ++jj) {
-          if (lane_ok && gi * RG + jj < r) f[jj].load(vp + coef_offset(r, n8, s0, gi * RG + jj));
+          if (lane_ok && gi * RG + jj < r) src.load(f[jj], 1, r, b0, qb0, n8, s0, gi * RG + jj);
           else f[jj].zero();
         }
         float pv[32];
@@ -326,8 +398,9 @@ void launch_decode_t(const Shape& s, const varrate_packed& c, const void* basis_
                      const void* q, int layer, const void* tail_k, const void* tail_v, int n_tail,
                      void* out, float* qt, float* part, int S, cudaStream_t st) {
   decode_rotate_kernel<T><<<dim3(s.G, s.B), 256, 0, st>>>((const T*)q, (const T*)basis_k, qt, s, layer);
-  decode_split_kernel<T, GP><<<dim3(S, s.G, s.B), 256, 0, st>>>((const T*)c.coef, c.bucket_count,
-                                                                c.bucket_base, qt, part, s, layer, S);
+  DenseSrc<T> src{(const T*)c.coef, c.bucket_base, s.cap, nullptr, nullptr};
+  decode_split_kernel<DenseSrc<T>, GP><<<dim3(S, s.G, s.B), 256, 0, st>>>(src, c.bucket_count, qt, part,
+                                                                           s, layer, S, 0);
   decode_combine_kernel<T, GP><<<dim3(s.G, s.B), 128, 0, st>>>(part, (const T*)q, (const T*)basis_v,
                                                                (const T*)tail_k, (const T*)tail_v,
                                                                n_tail, (T*)out, s, layer, S);
@@ -346,6 +419,26 @@ void dispatch_gp(int gp, const Shape& s, const varrate_packed& c, const void* bk
 }
 
 int group_pad(int grp) { return grp <= 1 ? 1 : grp <= 2 ? 2 : grp <= 4 ? 4 : 8; }
+
+template <int GP>
+void launch_decode_qt(const Shape& s, const varrate_qpacked& c, const void* basis_k, const void* basis_v,
+                      const void* q, int layer, const void* tail_k, const void* tail_v, int n_tail,
+                      void* out, float* qt, float* part, int S, cudaStream_t st) {
+  using bf = __nv_bfloat16;
+  decode_rotate_kernel<bf><<<dim3(s.G, s.B), 256, 0, st>>>((const bf*)q, (const bf*)basis_k, qt, s, layer);
+  if (c.bits == 4) {
+    QuantSrc<4> src{c.data, c.qbase, c.qcap_bytes, nullptr, nullptr};
+    decode_split_kernel<QuantSrc<4>, GP><<<dim3(S, s.G, s.B), 256, 0, st>>>(src, c.bucket_count, qt, part,
+                                                                           s, layer, S, c.qcap_bytes);
+  } else {
+    QuantSrc<8> src{c.data, c.qbase, c.qcap_bytes, nullptr, nullptr};
+    decode_split_kernel<QuantSrc<8>, GP><<<dim3(S, s.G, s.B), 256, 0, st>>>(src, c.bucket_count, qt, part,
+                                                                           s, layer, S, c.qcap_bytes);
+  }
+  decode_combine_kernel<bf, GP><<<dim3(s.G, s.B), 128, 0, st>>>(part, (const bf*)q, (const bf*)basis_v,
+                                                               (const bf*)tail_k, (const bf*)tail_v,
+                                                               n_tail, (bf*)out, s, layer, S);
+}
 
 }  // namespace
 
@@ -386,6 +479,24 @@ int launch_decode(const Shape& s, const varrate_packed& cache, const void* basis
     dispatch_gp<__nv_bfloat16>(gp, s, cache, basis_k, basis_v, q, layer, tail_k, tail_v, n_tail, out, qt, part, S, st);
   else
     dispatch_gp<float>(gp, s, cache, basis_k, basis_v, q, layer, tail_k, tail_v, n_tail, out, qt, part, S, st);
+  return 3;
+}
+
+int launch_decode_q(const Shape& s, const varrate_qpacked& cache, const void* basis_k,
+                    const void* basis_v, const void* q, int layer, const void* tail_k,
+                    const void* tail_v, int n_tail, void* out, void* ws, int num_sms, cudaStream_t st) {
+  ws = static_cast<char*>(ws) + kDecodeCounterBytes;   // same scratch layout as the general path
+  const int S = decode_splits(s, num_sms);
+  float* qt = reinterpret_cast<float*>(ws);
+  size_t a = (size_t)s.B * s.H * kHeadDim * sizeof(float);
+  a = (a + 255) & ~size_t(255);
+  float* part = reinterpret_cast<float*>(static_cast<char*>(ws) + a);
+  switch (group_pad(s.grp)) {
+    case 1: launch_decode_qt<1>(s, cache, basis_k, basis_v, q, layer, tail_k, tail_v, n_tail, out, qt, part, S, st); break;
+    case 2: launch_decode_qt<2>(s, cache, basis_k, basis_v, q, layer, tail_k, tail_v, n_tail, out, qt, part, S, st); break;
+    case 4: launch_decode_qt<4>(s, cache, basis_k, basis_v, q, layer, tail_k, tail_v, n_tail, out, qt, part, S, st); break;
+    default: launch_decode_qt<8>(s, cache, basis_k, basis_v, q, layer, tail_k, tail_v, n_tail, out, qt, part, S, st); break;
+  }
   return 3;
 }
 

@@ -68,4 +68,11 @@ int launch_decode(const Shape& s, const varrate_packed& cache, const void* basis
                   const void* tail_v, int n_tail, void* out, int32_t* dev_status, void* ws,
                   int num_sms, cudaStream_t st);
 
+// ---- quantized coefficients (quant.cu; decode with the general kernels in decode.cu)
+int launch_quantize(const Shape& s, const varrate_packed& in, const varrate_qpacked& out,
+                    int32_t* dev_status, cudaStream_t st);
+int launch_decode_q(const Shape& s, const varrate_qpacked& cache, const void* basis_k,
+                    const void* basis_v, const void* q, int layer, const void* tail_k,
+                    const void* tail_v, int n_tail, void* out, void* ws, int num_sms, cudaStream_t st);
+
 }  // namespace vr

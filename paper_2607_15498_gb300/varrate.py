@@ -56,6 +56,11 @@ class varrate_packed(ctypes.Structure):
                 ("cap_elems", ctypes.c_int64)]
 
 
+class varrate_qpacked(ctypes.Structure):
+    _fields_ = [("data", _c_void_p), ("qbase", _c_void_p), ("bucket_count", _c_void_p),
+                ("bits", ctypes.c_int32), ("qcap_bytes", ctypes.c_int64)]
+
+
 _lib = None
 
 _SIGS = {
@@ -81,6 +86,14 @@ _SIGS = {
                                              _c_void_p, ctypes.c_int32, _c_void_p, _c_void_p,
                                              ctypes.c_int32, _c_void_p, _c_void_p, _c_void_p,
                                              ctypes.c_size_t, _c_void_p]),
+    "varrate_qpacked_cap_bytes": (ctypes.c_int64, [ctypes.POINTER(varrate_config), ctypes.c_int32]),
+    "varrate_quantize": (ctypes.c_int32, [ctypes.POINTER(varrate_config), ctypes.POINTER(varrate_packed),
+                                          ctypes.POINTER(varrate_qpacked), _c_void_p, _c_void_p]),
+    "varrate_decode_attn_q": (ctypes.c_int32, [ctypes.POINTER(varrate_config),
+                                               ctypes.POINTER(varrate_qpacked), _c_void_p, _c_void_p,
+                                               _c_void_p, ctypes.c_int32, _c_void_p, _c_void_p,
+                                               ctypes.c_int32, _c_void_p, _c_void_p, _c_void_p,
+                                               ctypes.c_size_t, _c_void_p]),
     "varrate_decode_attn_noalloc": (ctypes.c_int32, [ctypes.POINTER(varrate_config),
                                                      ctypes.POINTER(varrate_packed), _c_void_p,
                                                      _c_void_p, _c_void_p, ctypes.c_int32,
@@ -209,6 +222,23 @@ def varrate_decode_attn_noalloc(cfg, packed, basis_k, basis_v, q, layer, tail_k,
                                              _ptr(dev_status), _stream(stream))
 
 
+def varrate_qpacked_cap_bytes(cfg: varrate_config, bits: int) -> int:
+    return lib().varrate_qpacked_cap_bytes(ctypes.byref(cfg), bits)
+
+
+def varrate_quantize(cfg, packed, qpacked, dev_status, stream=None) -> int:
+    return lib().varrate_quantize(ctypes.byref(cfg), ctypes.byref(packed.c), ctypes.byref(qpacked.c),
+                                  _ptr(dev_status), _stream(stream))
+
+
+def varrate_decode_attn_q(cfg, qpacked, basis_k, basis_v, q, layer, tail_k, tail_v, n_tail, out,
+                          dev_status, ws, stream=None) -> int:
+    return lib().varrate_decode_attn_q(ctypes.byref(cfg), ctypes.byref(qpacked.c), _ptr(basis_k),
+                                       _ptr(basis_v), _ptr(q), layer, _ptr(tail_k), _ptr(tail_v),
+                                       n_tail, _ptr(out), _ptr(dev_status), _ptr(ws), _nbytes(ws),
+                                       _stream(stream))
+
+
 # ------------------------------------------------------------- device-memory plumbing
 
 def make_config(n_layers, n_kv_heads, group, n_ctx, batch=1, budget_frac=0.2, r_min=16, window=32,
@@ -253,6 +283,29 @@ class PackedCache:
     def nbytes(self) -> int:
         return sum(t.numel() * t.element_size() for t in
                    (self.coef, self.bucket_count, self.bucket_base, self.perm, self.pos, self.ranks))
+
+
+@dataclass
+class QPackedCache:
+    """Torch-allocated buffers of a quantized cache (codes and group parameters, bucket byte
+    offsets) plus the C struct; the bucket counts are those of the source PackedCache."""
+    data: torch.Tensor
+    qbase: torch.Tensor
+    source: PackedCache
+    bits: int
+    qcap_bytes: int
+    c: varrate_qpacked
+
+    @staticmethod
+    def allocate(cfg: varrate_config, source: PackedCache, bits: int, device="cuda") -> "QPackedCache":
+        cap = varrate_qpacked_cap_bytes(cfg, bits)
+        if cap < 0:
+            raise VarrateError(ERR_ARG, "varrate_qpacked_cap_bytes")
+        B, L, G, d = cfg.batch, cfg.n_layers, cfg.n_kv_heads, cfg.head_dim
+        data = torch.zeros((B, L, G, 2, cap), dtype=torch.uint8, device=device)
+        qbase = torch.zeros((B, L, d + 2), dtype=torch.int64, device=device)
+        c = varrate_qpacked(data.data_ptr(), qbase.data_ptr(), source.bucket_count.data_ptr(), bits, cap)
+        return QPackedCache(data, qbase, source, bits, cap, c)
 
 
 def workspace(cfg: varrate_config, which_call: int, device="cuda") -> torch.Tensor:

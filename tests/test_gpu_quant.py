@@ -1,0 +1,220 @@
+"""GPU parity of the coefficient quantization (group-wise b-bit, Sec. 3.3 "Composability") and of
+decode attention on the quantized cache, through the C ABI.
+
+The device cache is built from the oracle: its per-token coefficients (rounded to bf16, the stored
+precision) and bucket tables are written into the packed layout by a test helper, so both sides
+quantize the same values. Bars: codes, group offsets and steps and the bucket byte offsets
+bit-exact; decode within the decode bars of gpu_helpers (max-abs 2e-2 and, per row, 2^-6 of the
+row's largest magnitude) against the oracle's decode on its own dequantized coefficients."""
+import numpy as np
+import pytest
+import torch
+
+from gpu_helpers import (O, V, cfg_for, coef_index, decode_close, decode_errors, f64, oracle_layer,
+                         synth)
+
+pytestmark = pytest.mark.gpu
+
+CASES = {
+    "llama_ragged": synth.workload("llama1", n_kv_heads=2, n_ctx=4096 + 37, batch=2, n_layers=2),
+    "qwen_g7": synth.workload("qwen", n_kv_heads=2, n_ctx=3000 + 5, n_layers=1),
+}
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _gpu(vlib):
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA GPU")
+
+
+def _bf16(x):
+    return torch.as_tensor(np.asarray(x, dtype=np.float64)).to(torch.bfloat16).to(torch.float64).numpy()
+
+
+def _write_stream(buf, coef, ranks, count, base, pos):
+    """Lay the (bf16-valued) coefficients of one stream into a packed buffer (packed layout)."""
+    ranks = np.asarray(ranks, dtype=np.int64)
+    n8 = (np.asarray(count, dtype=np.int64) + 7) // 8 * 8
+    j = np.arange(128)[None, :]
+    rr = ranks[:, None]
+    idx = coef_index(np.asarray(base)[rr], rr, n8[rr], np.asarray(pos, dtype=np.int64)[:, None], j)
+    mask = j < rr
+    buf[idx[mask]] = coef[mask]
+
+
+def oracle_cache(wl, refs, cfg, pairs):
+    """A device PackedCache holding, for the given (b, l) pairs, the oracle's tables and its
+    coefficients rounded to bf16; returns it with the bf16 coefficients per pair [G][2][N][d]."""
+    packed = V.PackedCache.allocate(cfg, "cuda")
+    coefs = {}
+    for (b, l) in pairs:
+        ref = refs[(b, l)]
+        packed.bucket_count[b, l].copy_(torch.as_tensor(ref["count"]))
+        packed.bucket_base[b, l].copy_(torch.as_tensor(ref["base"]))
+        packed.pos[b, l].copy_(torch.as_tensor(ref["pos"]))
+        packed.perm[b, l].copy_(torch.as_tensor(ref["perm"]))
+        packed.ranks[b, l].copy_(torch.as_tensor(ref["ranks"].astype(np.uint8)))
+        c16 = np.stack([np.stack([_bf16(O.truncate(ref[k][g], ref["ranks"])) for k in ("coef_k", "coef_v")])
+                        for g in range(wl.n_kv_heads)])
+        coefs[(b, l)] = c16
+        for g in range(wl.n_kv_heads):
+            for kv in range(2):
+                buf = np.zeros(packed.cap_elems)
+                _write_stream(buf, c16[g, kv], ref["ranks"], ref["count"], ref["base"], ref["pos"])
+                packed.coef[b, l, g, kv].copy_(torch.as_tensor(buf).to(torch.bfloat16))
+    return packed, coefs
+
+
+def read_quantized(qp, b, l, g, kv, ranks, count, pos, bits):
+    """Codes [N][d] and group (offset, step) [N][d] read from the device buffer by the layout of
+    include/varrate.h (zero beyond each rank)."""
+    data = qp.data[b, l, g, kv].cpu().numpy()
+    qbase = qp.qbase[b, l].cpu().numpy()
+    ranks = np.asarray(ranks, dtype=np.int64)
+    n = ranks.size
+    codes = np.zeros((n, 128), np.uint8)
+    lo = np.zeros((n, 128), np.float16)
+    st = np.zeros((n, 128), np.float16)
+    full = O.qrow_bytes(128, bits)
+    for t in range(n):
+        r, p = int(ranks[t]), int(pos[t])
+        n8 = (int(count[r]) + 7) // 8 * 8
+        i, pl = p // 128, p % 128
+        tl = min(128, n8 - 128 * i)
+        for j in range(r):
+            row = int(qbase[r]) + i * r * full + j * O.qrow_bytes(tl, bits)
+            if bits == 4:
+                byte = data[row + pl // 2]
+                codes[t, j] = (byte >> 4) if (pl & 1) else (byte & 15)
+            else:
+                codes[t, j] = data[row + pl]
+            par = data[row + tl * bits // 8 + 4 * (pl // 32): row + tl * bits // 8 + 4 * (pl // 32) + 4]
+            lo[t, j], st[t, j] = par.view(np.float16)
+    return codes, lo, st
+
+
+def _setup(name):
+    wl = CASES[name]
+    k, v, qw, bk, bv = synth.stack_inputs(wl)
+    cfg = cfg_for(wl)
+    pairs = [(b, l) for b in range(wl.batch) for l in range(wl.n_layers)]
+    refs = {(b, l): oracle_layer(wl, k, v, qw, bk, bv, b, l) for (b, l) in pairs}
+    packed, coefs = oracle_cache(wl, refs, cfg, pairs)
+    return wl, cfg, bk, bv, refs, packed, coefs, pairs
+
+
+@pytest.mark.parametrize("bits", [4, 8])
+@pytest.mark.parametrize("name", list(CASES))
+def test_quantize_bit_exact(name, bits):
+    wl, cfg, bk, bv, refs, packed, coefs, pairs = _setup(name)
+    qp = V.QPackedCache.allocate(cfg, packed, bits)
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    V.check(V.varrate_quantize(cfg, packed, qp, status), "varrate_quantize")
+    torch.cuda.synchronize()
+    assert int(status.item()) == V.OK
+    for (b, l) in pairs:
+        ref = refs[(b, l)]
+        qb = O.qpack_tables(ref["count"], wl.r_min, wl.head_dim, bits)
+        np.testing.assert_array_equal(qp.qbase[b, l].cpu().numpy(), qb)
+        assert qb[-1] <= qp.qcap_bytes
+        for g in range(wl.n_kv_heads):
+            for kv in range(2):
+                want = O.quantize_coefficients(coefs[(b, l)][g, kv], ref["ranks"], ref["count"],
+                                               ref["pos"], bits)
+                codes, lo, st = read_quantized(qp, b, l, g, kv, ref["ranks"], ref["count"],
+                                               ref["pos"], bits)
+                mask = np.arange(128)[None, :] < ref["ranks"][:, None]
+                np.testing.assert_array_equal(codes[mask], want[0][mask])
+                np.testing.assert_array_equal(lo[mask].view(np.uint16), want[1][mask].view(np.uint16))
+                np.testing.assert_array_equal(st[mask].view(np.uint16), want[2][mask].view(np.uint16))
+
+
+@pytest.mark.parametrize("bits,n_tail", [(4, 0), (8, 0), (4, 37)])
+@pytest.mark.parametrize("name", list(CASES))
+def test_decode_on_quantized_cache(name, bits, n_tail):
+    wl, cfg, bk, bv, refs, packed, coefs, pairs = _setup(name)
+    qp = V.QPackedCache.allocate(cfg, packed, bits)
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    V.check(V.varrate_quantize(cfg, packed, qp, status), "varrate_quantize")
+    ws = V.workspace(cfg, V.CALL_DECODE)
+    gen = torch.Generator().manual_seed(11)
+    worst = (0.0, 0.0)
+    for l in range(wl.n_layers):
+        q = synth.stack_decode_queries(wl, l, 1)[0]
+        tk = tv = None
+        if n_tail:
+            shape = (wl.batch, wl.n_kv_heads, n_tail, wl.head_dim)
+            tk = torch.randn(shape, generator=gen).to(torch.bfloat16)
+            tv = torch.randn(shape, generator=gen).to(torch.bfloat16)
+        out = torch.empty_like(q, device="cuda")
+        V.check(V.varrate_decode_attn_q(cfg, qp, bk.cuda(), bv.cuda(), q.cuda(), l,
+                                        None if tk is None else tk.cuda(),
+                                        None if tv is None else tv.cuda(), n_tail, out, status, ws),
+                "varrate_decode_attn_q")
+        torch.cuda.synchronize()
+        assert int(status.item()) == V.OK
+        got = f64(out)
+        for b in range(wl.batch):
+            ref = refs[(b, l)]
+            deq = [[O.quantize_coefficients(coefs[(b, l)][g, kv], ref["ranks"], ref["count"],
+                                            ref["pos"], bits)[3] for g in range(wl.n_kv_heads)]
+                   for kv in range(2)]
+            want = O.decode_coef(f64(q[b]), np.stack(deq[0]).astype(np.float64),
+                                 np.stack(deq[1]).astype(np.float64), ref["ranks"], f64(bk[l]),
+                                 f64(bv[l]), None if tk is None else f64(tk[b]),
+                                 None if tv is None else f64(tv[b]))
+            assert decode_close(got[b], want, cfg), (l, b, decode_errors(got[b], want))
+            worst = tuple(max(a, e) for a, e in zip(worst, decode_errors(got[b], want)))
+    print(f"{name} {bits}-bit: decode worst relative / absolute error {worst[0]:.3e} / {worst[1]:.3e}")
+
+
+def test_quantized_round_trip_bound_at_full_size():
+    """llama32 layer call (8 sequences x 8 KV heads x N = 32768, GPU encode): every quantized group
+    reproduces the stored coefficients within half a step plus the fp16 rounding of its offset
+    (a property of the definition at any size); the quantized streams are ~32% (4-bit) and ~57%
+    (8-bit) of the bf16 ones."""
+    wl = synth.workload("llama32", n_layers=1)
+    k, v, qw, bk, bv = synth.stack_inputs(wl, device="cuda")
+    cfg = cfg_for(wl)
+    packed = V.PackedCache.allocate(cfg, "cuda")
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    V.check(V.varrate_encode(cfg, qw, k, v, bk, bv, None, packed, None, status,
+                             V.workspace(cfg, V.CALL_ENCODE)))
+    del k, v, qw
+    for bits in (4, 8):
+        qp = V.QPackedCache.allocate(cfg, packed, bits)
+        V.check(V.varrate_quantize(cfg, packed, qp, status))
+        torch.cuda.synchronize()
+        assert int(status.item()) == V.OK
+        counts = packed.bucket_count.cpu().numpy()
+        for b in (0, 7):
+            ref_base = packed.bucket_base[b, 0].cpu().numpy()
+            qb = O.qpack_tables(counts[b, 0], wl.r_min, wl.head_dim, bits)
+            np.testing.assert_array_equal(qp.qbase[b, 0].cpu().numpy(), qb)
+            # bytes per coefficient: (b + 1) / 8 against 2 in bf16, plus short-tile rounding
+            ratio = qb[-1] / (2.0 * ref_base[-1])
+            assert (0.3125 if bits == 4 else 0.5625) <= ratio < (0.34 if bits == 4 else 0.59), ratio
+            # one stream: dequantize every row of every tile and compare with the bf16 coefficients
+            g, kv = 5, 1
+            data = qp.data[b, 0, g, kv].cpu().numpy()
+            src = packed.coef[b, 0, g, kv].to(torch.float32).cpu().numpy()
+            full = O.qrow_bytes(128, bits)
+            for r in range(wl.r_min, wl.head_dim + 1):
+                n8 = (int(counts[b, 0, r]) + 7) // 8 * 8
+                for t0 in range(0, n8, 128):
+                    tl = min(128, n8 - t0)
+                    for j in range(r):
+                        row = int(qb[r]) + (t0 // 128) * r * full + j * O.qrow_bytes(tl, bits)
+                        raw = data[row: row + tl * bits // 8]
+                        codes = (np.stack([raw & 15, raw >> 4], 1).reshape(-1) if bits == 4 else raw)
+                        par = data[row + tl * bits // 8: row + tl * bits // 8 + 4 * ((tl + 31) // 32)].view(np.float16)
+                        lo32, st32 = par[0::2].astype(np.float32), par[1::2].astype(np.float32)
+                        grp = np.arange(tl) // 32
+                        xh = (lo32[grp] + (codes.astype(np.float32) * st32[grp]).astype(np.float32)).astype(np.float32)
+                        # bf16 row j of the tile: 8-slot group p at position (p + j) mod (tl / 8)
+                        off = int(ref_base[r]) + t0 * r + j * tl
+                        ng = tl // 8
+                        x = src[off: off + tl].reshape(ng, 8)[(np.arange(ng) + j) % ng].reshape(-1)
+                        xmax = np.abs(x.reshape(-1, 8)).max()
+                        bound = 0.5 * st32[grp] + 2.0 ** -10 * max(xmax, 1e-30)
+                        assert np.all(np.abs(xh - x) <= bound), (bits, r, t0, j)
