@@ -420,9 +420,11 @@ def sweep_config(V, wl, dev, peak, stream, decode_steps, copies=1, flush=False, 
 
 def sweep_reuse(V, wl, dev, peak, stream, n_batches, n_window, n_decode):
     """Long-context reuse: encode once, then `n_batches` seeded query batches, each `n_window`
-    window steps followed by `n_decode` decode steps. Every step appends its token to the exact
-    tail (step i decodes with n_tail = i + 1 exact tokens after the cache) and runs one decode
-    call per layer; all batches read the same packed cache."""
+    window tokens followed by `n_decode` decode steps, all reading the same packed cache. The
+    window runs as one window-decode call per layer (varrate_decode_window: query i sees the
+    cache and the exact tail up to its own token), and, for comparison, as `n_window` single-query
+    calls per layer (step i with n_tail = i + 1). Decode step i appends its token to the exact tail
+    and runs one single-query call per layer (n_tail = n_window + i + 1)."""
     cfg = V.make_config(wl.n_layers, wl.n_kv_heads, wl.group, wl.n_ctx, batch=wl.batch,
                         budget_frac=wl.budget_frac, r_min=wl.r_min, window=wl.window, dtype=V.BF16)
     k, v, qw, bk, bv = synth.stack_inputs(wl, device=dev)
@@ -431,6 +433,7 @@ def sweep_reuse(V, wl, dev, peak, stream, n_batches, n_window, n_decode):
     status = torch.zeros(1, dtype=torch.int32, device=dev)
     ws_enc = V.workspace(cfg, V.CALL_ENCODE, dev)
     ws_dec = V.workspace(cfg, V.CALL_DECODE, dev)
+    ws_win = V.workspace(cfg, V.CALL_DECODE_WINDOW, dev)
     enc = []
     for i in range(3):
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -445,61 +448,82 @@ def sweep_reuse(V, wl, dev, peak, stream, n_batches, n_window, n_decode):
     del k, v, qw
     torch.cuda.empty_cache()
     n_steps = n_window + n_decode
-    d, G = wl.head_dim, wl.n_kv_heads
+    d, G, H = wl.head_dim, wl.n_kv_heads, wl.n_q_heads
     per_layer = coded_bytes_per_layer(packed, cfg)
-    fixed = 2 * G * d * d * 2 + 2 * wl.batch * wl.n_q_heads * d * 2
-    out = torch.empty((wl.batch, wl.n_q_heads, d), dtype=torch.bfloat16, device=dev)
+    fixed = 2 * G * d * d * 2 + 2 * wl.batch * H * d * 2
+    out = torch.empty((wl.batch, H, d), dtype=torch.bfloat16, device=dev)
+    out_w = torch.empty((wl.batch, n_window, H, d), dtype=torch.bfloat16, device=dev)
     status.zero_()
-    total_ms, total_bytes, win_ms = 0.0, 0, []
+    win_ms, seq_ms, dec_ms = [], [], []
     for qb in range(n_batches + 1):                 # batch 0 is a warm-up
         gen = torch.Generator(device=dev)
         gen.manual_seed(synth.seed_of(wl, "qdec", 0, 0, 0, 1000 + qb))
-        q = torch.randn((n_steps, wl.n_layers, wl.batch, wl.n_q_heads, d), generator=gen,
+        q = torch.randn((n_steps, wl.n_layers, wl.batch, H, d), generator=gen,
                         device=dev).to(torch.bfloat16)
         tk = torch.randn((wl.n_layers, wl.batch, G, n_steps, d), generator=gen, device=dev).to(torch.bfloat16)
         tv = torch.randn((wl.n_layers, wl.batch, G, n_steps, d), generator=gen, device=dev).to(torch.bfloat16)
         # the tail of step i is the first i + 1 rows: one contiguous [B][G][i + 1][d] block per layer
         tails = [[(tk[l, :, :, : i + 1].contiguous(), tv[l, :, :, : i + 1].contiguous())
                   for l in range(wl.n_layers)] for i in range(n_steps)]
-        def window(lo, hi):
+        qwin = [q[:n_window, l].permute(1, 0, 2, 3).contiguous() for l in range(wl.n_layers)]
+
+        def steps(lo, hi):
             for i in range(lo, hi):
                 for l in range(wl.n_layers):
                     a, b_ = tails[i][l]
                     V.check(V.varrate_decode_attn(cfg, packed, bk, bv, q[i, l], l, a, b_, i + 1,
                                                   out, status, ws_dec, None), "varrate_decode_attn")
+
+        def window_calls():
+            for l in range(wl.n_layers):
+                a, b_ = tails[n_window - 1][l]
+                V.check(V.varrate_decode_window(cfg, packed, bk, bv, qwin[l], n_window, l, a, b_,
+                                                n_window, out_w, status, ws_win, None),
+                        "varrate_decode_window")
         if qb == 0:
-            window(0, n_steps)          # first calls on this workspace: outside capture
-        gw = capture(lambda: window(0, n_window))
-        gd = capture(lambda: window(n_window, n_steps))
-        ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+            steps(0, n_steps)          # first calls on these workspaces: outside capture
+            window_calls()
+        gwin = capture(window_calls)
+        gseq = capture(lambda: steps(0, n_window))
+        gdec = capture(lambda: steps(n_window, n_steps))
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
         ev[0].record(stream)
-        gw.replay()
+        gwin.replay()
         ev[1].record(stream)
-        gd.replay()
+        gdec.replay()
         ev[2].record(stream)
+        gseq.replay()
+        ev[3].record(stream)
         torch.cuda.synchronize()
-        del gw, gd
+        del gwin, gseq, gdec
         if qb > 0:
-            total_ms += ev[0].elapsed_time(ev[2])
             win_ms.append(ev[0].elapsed_time(ev[1]))
-            tail_bytes = sum(2 * wl.batch * G * (i + 1) * d * 2 for i in range(n_steps))
-            total_bytes += n_steps * (sum(per_layer) + wl.n_layers * fixed) + wl.n_layers * tail_bytes
-        del tails, tk, tv, q
-    gbs = total_bytes / (total_ms * 1e-3) / 1e9
-    n_calls = n_batches * n_steps * wl.n_layers
+            dec_ms.append(ev[1].elapsed_time(ev[2]))
+            seq_ms.append(ev[2].elapsed_time(ev[3]))
+        del tails, tk, tv, q, qwin
+    # algorithmic bytes: the coefficients, bases, queries and outputs of every call, and its tail
+    dec_bytes = n_decode * (sum(per_layer) + wl.n_layers * fixed) + wl.n_layers * sum(
+        2 * wl.batch * G * (i + 1) * d * 2 for i in range(n_window, n_steps))
+    win_fixed = 2 * G * d * d * 2 + 2 * wl.batch * n_window * H * d * 2
+    win_bytes = sum(per_layer) + wl.n_layers * (win_fixed + 2 * wl.batch * G * n_window * d * 2)
+    dec_gbs = dec_bytes / (statistics.mean(dec_ms) * 1e-3) / 1e9
+    win_gbs = win_bytes / (statistics.mean(win_ms) * 1e-3) / 1e9
     return {"workload": workload_desc(wl) + f"; {n_batches} query batches of {n_window} window + "
-                                              f"{n_decode} decode steps, exact tail growing 1..{n_steps}",
+                                              f"{n_decode} decode tokens, exact tail growing to {n_steps}",
             "encode_ms_per_layer": round(statistics.median(enc) / wl.n_layers, 4),
             "encode_ms_per_32k_ctx": round(statistics.median(enc) / wl.batch * 32768 / wl.n_ctx, 4),
             "encode_status": V.status_string(enc_status),
-            "decode_gbs": round(gbs, 1), "decode_frac_of_hbm_peak": round(gbs / peak, 4),
-            "decode_us_per_layer_call": round(total_ms * 1e3 / n_calls, 2),
-            "decode_bytes_per_layer_call": int(total_bytes / n_calls),
+            "decode_gbs": round(dec_gbs, 1), "decode_frac_of_hbm_peak": round(dec_gbs / peak, 4),
+            "decode_us_per_layer_call": round(statistics.mean(dec_ms) * 1e3 / (n_decode * wl.n_layers), 2),
+            "decode_bytes_per_layer_call": int(dec_bytes / (n_decode * wl.n_layers)),
             "window_ms_per_batch": round(statistics.mean(win_ms), 3),
-            "ms_per_query_batch": round(total_ms / n_batches, 3),
+            "window_us_per_layer_call": round(statistics.mean(win_ms) * 1e3 / wl.n_layers, 2),
+            "window_gbs": round(win_gbs, 1), "window_frac_of_hbm_peak": round(win_gbs / peak, 4),
+            "window_ms_per_batch_as_single_query_calls": round(statistics.mean(seq_ms), 3),
+            "ms_per_query_batch": round(statistics.mean(win_ms) + statistics.mean(dec_ms), 3),
             "decode_status": V.status_string(int(status.item())),
-            "decode_issue": "per query batch, CUDA graphs of its window steps and of its decode "
-                            "steps (one captured call per layer and step)",
+            "decode_issue": "per query batch, CUDA graphs of its window calls (one per layer), of "
+                            "its decode steps and of the window as single-query steps",
             "l2": "packed cache of all layers (3.4 GB) read per step (> L2)"}
 
 

@@ -13,9 +13,9 @@
  *    PyTorch allocations are); a misaligned pointer is VARRATE_ERR_ARG. The library never
  *    allocates or frees device memory. Calls are reentrant and thread-safe. Across calls the
  *    library keeps only per-process values that do not change results: each device's SM count,
- *    the driver entry point that encodes TMA descriptors, a counter that tags every decode call
- *    (see varrate_decode_attn), and the device address of the allocation-free entry point's
- *    scratch array. All are held in atomics.
+ *    the driver entry point that encodes TMA descriptors, whether a kernel's shared-memory opt-in
+ *    was made on a device, and the device address of the allocation-free entry point's scratch
+ *    array. All are held in atomics.
  *  - `stream` is a cudaStream_t passed as void* (NULL = the legacy default stream). Every call
  *    only enqueues work on `stream` and returns without synchronising.
  *  - The return value reports what the host can see: bad arguments (VARRATE_ERR_ARG), a workspace
@@ -132,7 +132,8 @@ typedef enum {
   VARRATE_CALL_SALIENCE = 0,
   VARRATE_CALL_PACK = 1,
   VARRATE_CALL_ENCODE = 2,
-  VARRATE_CALL_DECODE = 3
+  VARRATE_CALL_DECODE = 3,
+  VARRATE_CALL_DECODE_WINDOW = 4
 } varrate_call;
 
 /* Library version (major * 10000 + minor * 100 + patch). */
@@ -227,6 +228,29 @@ varrate_status varrate_decode_attn(const varrate_config* cfg, const varrate_pack
                                    int32_t layer, const void* tail_k, const void* tail_v,
                                    int32_t n_tail, void* out, int32_t* dev_status, void* ws,
                                    size_t ws_bytes, void* stream);
+
+/* Step 4 for a window of new tokens — decode attention of n_q consecutive queries per sequence in
+ * one call (the multi-token form of varrate_decode_attn: speculative or chunked decoding). The last
+ * n_q tokens of the exact tail are the window; query i (0 <= i < n_q) sits at tail position
+ * n_tail - n_q + i and, as in causal attention (Sec. 3.1), attends to every coded token and to the
+ * tail tokens 0 .. n_tail - n_q + i. Per query head h of KV head g the result is that of
+ * varrate_decode_attn for query i with the tail cut after its own position.
+ *   q         [B][n_q][H][d] bf16
+ *   tail_k/_v [B][G][n_tail][d] bf16, n_q <= n_tail <= 4096
+ *   out       [B][n_q][H][d] bf16
+ *   ws        at least varrate_workspace_bytes(cfg, VARRATE_CALL_DECODE_WINDOW) bytes: scratch that
+ *             a call writes before it reads (no state is kept between calls; no zero-fill needed).
+ *             Calls that overlap on one workspace race.
+ * Limits: dtype VARRATE_BF16, batch <= 64, 1 <= n_q and n_q * group <= 128 (VARRATE_ERR_UNSUPPORTED
+ * otherwise; n_q > n_tail is VARRATE_ERR_ARG). Three kernels run (query rotation into MMA fragments,
+ * the coded part over the persistent grid, merge + causal tail + back-rotation), each launched
+ * with programmatic stream serialization; the same rule as for varrate_decode_attn applies to a
+ * following kernel launched with that attribute. */
+varrate_status varrate_decode_window(const varrate_config* cfg, const varrate_packed* cache,
+                                     const void* basis_k, const void* basis_v, const void* q,
+                                     int32_t n_q, int32_t layer, const void* tail_k,
+                                     const void* tail_v, int32_t n_tail, void* out,
+                                     int32_t* dev_status, void* ws, size_t ws_bytes, void* stream);
 
 /* Upper bound on the bytes of one quantized stream for any allocation within the budget:
  * with S = max(B_c, r_min * (N - w)) + w * d, R = sum_{r = r_min..d} r and F = qrow(128):

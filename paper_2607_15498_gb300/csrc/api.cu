@@ -86,6 +86,7 @@ size_t ws_bytes(const varrate_config* c, int32_t which) {
       return vr::salience_ws_bytes(s, sms) + align256((size_t)s.B * s.L * s.n_coded * sizeof(float)) +
              align256((size_t)s.B * s.L * sizeof(int64_t));
     case VARRATE_CALL_DECODE: return vr::decode_ws_bytes(s, sms);
+    case VARRATE_CALL_DECODE_WINDOW: return vr::decode_window_ws_bytes(s, sms);
     default: return 0;
   }
 }
@@ -250,6 +251,29 @@ varrate_status varrate_decode_attn(const varrate_config* cfg, const varrate_pack
   const Shape s = make_shape(cfg, cache->cap_elems);
   if (vr::launch_decode(s, *cache, basis_k, basis_v, q, layer, tail_k, tail_v, n_tail, out, dev_status,
                         ws, num_sms(), (cudaStream_t)stream) < 0)
+    return VARRATE_ERR_CUDA;
+  return launched();
+}
+
+varrate_status varrate_decode_window(const varrate_config* cfg, const varrate_packed* cache,
+                                     const void* basis_k, const void* basis_v, const void* q,
+                                     int32_t n_q, int32_t layer, const void* tail_k,
+                                     const void* tail_v, int32_t n_tail, void* out,
+                                     int32_t* dev_status, void* ws, size_t ws_bytes_, void* stream) {
+  varrate_status st = check(cfg);
+  if (st != VARRATE_OK) return st;
+  if (cfg->dtype != VARRATE_BF16) return VARRATE_ERR_UNSUPPORTED;
+  if (!packed_ok(cfg, cache) || !basis_k || !basis_v || !q || !out || !tail_k || !tail_v)
+    return VARRATE_ERR_ARG;
+  if (layer < 0 || layer >= cfg->n_layers || n_q < 1 || n_tail < n_q) return VARRATE_ERR_ARG;
+  if (n_tail > 4096) return VARRATE_ERR_UNSUPPORTED;
+  if (!aligned16({basis_k, basis_v, q, tail_k, tail_v, out, dev_status, ws})) return VARRATE_ERR_ARG;
+  const Shape s = make_shape(cfg, cache->cap_elems);
+  if (!vr::decode_window_supported(s, n_q, n_tail, num_sms())) return VARRATE_ERR_UNSUPPORTED;
+  const size_t need = ws_bytes(cfg, VARRATE_CALL_DECODE_WINDOW);
+  if (ws_bytes_ < need || ws == nullptr) return VARRATE_ERR_WORKSPACE;
+  if (vr::launch_decode_window(s, *cache, basis_k, basis_v, q, n_q, layer, tail_k, tail_v, n_tail, out,
+                               dev_status, ws, num_sms(), (cudaStream_t)stream) < 0)
     return VARRATE_ERR_CUDA;
   return launched();
 }

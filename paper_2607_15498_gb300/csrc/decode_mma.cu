@@ -27,7 +27,7 @@
 //   values   O~^T[j][head] += V[j][slot] * P^T[slot][head]      (P in bf16, <= 2^-9 relative per
 //            weight, transposed from the score fragments with movmatrix)
 // Partials (max, sum, o~[128]) per (segment, CTA) go to the workspace. The last CTA to finish a
-// segment (counted in a per-segment completion word in the workspace, tagged with the call's epoch)
+// segment (counted in per-segment arrival counters in the workspace header, DecodeHeader below)
 // merges its partials, adds the exact tail, rotates back with U_V^T (staged in the idle ring) and
 // normalises, so one launch does the whole step.
 //
@@ -39,43 +39,17 @@
 #include <atomic>
 
 #include "common.cuh"
+#include "decode_common.cuh"
 #include "kernels.h"
 
 namespace vr {
 
 namespace {
 
-constexpr int kMaxR = kHeadDim;
 constexpr int NW = 8;                 // warps per CTA
 constexpr int ST = 3;                 // ring stages per warp
-constexpr int ISL = 128;              // slots per item
-constexpr int CH = 32;                // coefficient rows per chunk of a full 128-slot tile
-constexpr int STAGE = CH * ISL * 2;   // one chunk: up to 32 rows of a 128-slot tile
 constexpr int kPartStride = kHeadDim + 4;   // o~[128], max, sum, pad: rows 16-byte aligned
 constexpr int kHeadsPad = 8;
-constexpr uint32_t kWaitTries = 1u << 22;   // bounded mbarrier polls (well over a second)
-constexpr float kSlack = 8.f;                // headroom of the running max, log2 units
-// Cost-line allowance per (sequence, KV head) segment, in K-stream elements: a CTA that enters a
-// segment pays its set-up (tables, query rotation, pipeline ramp, partial write, and for one CTA
-// the combine), about as long as streaming this many coefficients at a CTA's share of HBM
-// bandwidth, so ranges that straddle segments are shortened by that much.
-constexpr long long kSegCost = 90112;
-
-// A 64-bit integer division is a long instruction sequence (measured ~600 cycles here), so the
-// cost-line arithmetic avoids it. n / d for d < 2^16 by long division in 16-bit digits: four
-// 32-bit divisions.
-__device__ __forceinline__ unsigned long long udiv_small(unsigned long long n, uint32_t d) {
-  unsigned long long q = 0;
-  uint32_t r = 0;
-#pragma unroll
-  for (int sh = 48; sh >= 0; sh -= 16) {
-    const uint32_t cur = (r << 16) | (uint32_t)((n >> sh) & 0xFFFFu);   // r < d < 2^16
-    const uint32_t qd = cur / d;
-    r = cur - qd * d;
-    q = (q << 16) | qd;
-  }
-  return q;
-}
 
 struct SegSmem {
   alignas(16) uint32_t qfrag[kHeadDim / 16][32][4];   // per j-chunk, per lane: b0 hi, b1 hi, b0 lo, b1 lo (read as uint4)
@@ -93,60 +67,6 @@ struct Merge {
   float mx[kHeadsPad], l[kHeadsPad];
   float acc[NW][kHeadsPad][kHeadDim];
 };
-
-// Items of one CTA inside its cost range [lo, hi) of a stream, in (rank, slot) order: item k lies
-// in bucket r with it_pref[r] <= k < it_pref[r + 1] and is item it_lo[r] + (k - it_pref[r]) of that
-// bucket. Warp w takes items w, w + NW, w + 2 NW, ...
-__device__ __forceinline__ void bucket_range(const SegSmem& sm, int r, long long lo, long long hi,
-                                             long long& i0, long long& i1) {
-  const int n = sm.cnt[r];
-  if (n == 0) { i0 = i1 = 0; return; }
-  const long long n8 = pad8(n), b0 = sm.base[r];
-  const long long nit = (n8 + ISL - 1) / ISL;
-  // ceil(x / (128 r)) = ceil(ceil(x / 128) / r)
-  auto items_before = [&](long long x) -> long long {
-    if (x <= 0) return 0;
-    const unsigned long long a = ((unsigned long long)x + ISL - 1) / ISL;
-    if (a < (1ull << 31)) return (long long)(((uint32_t)a + (uint32_t)r - 1u) / (uint32_t)r);
-    return (long long)udiv_small(a + r - 1, (uint32_t)r);
-  };
-  i0 = items_before(lo - b0);
-  i1 = items_before(hi - b0);
-  if (i1 > nit) i1 = nit;
-  if (i0 > i1) i0 = i1;
-}
-
-struct Item {
-  int r;    // bucket (rank)
-  int it;   // item index inside the bucket
-};
-
-__device__ __forceinline__ Item item_at(const SegSmem& sm, int k);
-
-// Item k after item x = item k - NW (round-robin): NW further in the same bucket, else a search.
-__device__ __forceinline__ Item next_rr(const SegSmem& sm, Item x, int k) {
-  if (k < sm.it_pref[x.r + 1]) { x.it += NW; return x; }
-  return item_at(sm, k);
-}
-
-__device__ __forceinline__ Item item_at(const SegSmem& sm, int k) {
-  int lo = 0, hi = kMaxR + 1;   // it_pref[lo] <= k < it_pref[hi]
-  while (hi - lo > 1) {
-    const int mid = (lo + hi) >> 1;
-    if (sm.it_pref[mid] <= k) lo = mid; else hi = mid;
-  }
-  Item x;
-  x.r = lo;
-  x.it = sm.it_lo[lo] + (k - sm.it_pref[lo]);
-  return x;
-}
-
-// Rows per chunk of a tile of tl slots, as log2: as many rows as fill one 8 KB stage (32 rows of a
-// full 128-slot tile, 64 of a tile of at most 64 slots, all 128 of a tile of at most 32). The
-// sparse high-rank buckets end in short tiles; reading them in few chunks keeps their items from
-// being a chain of small, latency-bound copies.
-__device__ __forceinline__ int chunk_lg(int tl) { return tl > 64 ? 5 : (tl > 32 ? 6 : 7); }
-static_assert((ISL * 2) << 5 == STAGE, "a full tile's chunk fills a stage");
 
 // Producer cursor: which chunk of which item comes next in this warp's stream.
 struct Prod {
@@ -185,24 +105,10 @@ __device__ __forceinline__ bool issue_chunk(Prod& p, const SegSmem& sm, const __
     if (++p.phase == 2) {
       p.phase = 0;
       p.k += NW;
-      if (p.k < total) p.item = next_rr(sm, p.item, p.k);
+      if (p.k < total) p.item = next_rr<NW>(sm, p.item, p.k);
     }
   }
   return true;
-}
-
-// (x + 2) mod n for 0 <= x < n, n >= 1
-__device__ __forceinline__ int wrap2(int x, int n) {
-  x += 2;
-  x -= (x >= n) ? n : 0;
-  x -= (x >= n) ? n : 0;
-  return x;
-}
-
-// Keep the bf16 halves of `w` whose row index (lo half: j, hi half: j + 1) is below r.
-__device__ __forceinline__ uint32_t keep_rows(uint32_t w, int j, int r) {
-  const uint32_t m = (j < r ? 0x0000FFFFu : 0u) | (j + 1 < r ? 0xFFFF0000u : 0u);
-  return w & m;
 }
 
 // Rotate the queries of (b, g) into the basis: qt[head][j] = scale * sum_i U_K[j][i] q[head][i],
@@ -269,33 +175,6 @@ __device__ void build_qfrag(SegSmem& sm, int tid) {
   }
 }
 
-// Start of CTA c's range on a cost line of T elements cut into C equal ranges: floor(T c / C).
-// The launcher guarantees T * C < 2^63 and C <= kMaxCtas < 2^16.
-__device__ __forceinline__ long long cut_at(long long T, long long c, int C) {
-  return (long long)udiv_small((unsigned long long)T * (unsigned long long)c, (uint32_t)C);
-}
-
-// CTAs whose cost range [cuts[c], cuts[c + 1]) meets [P, P + W): c0..c1 (W > 0, P + W <= T,
-// cuts[c] = floor(T c / C)). c0 is the first c with cuts[c + 1] > P, i.e. ceil((P + 1) C / T) - 1,
-// and c1 + 1 the first c with cuts[c] > P + W - 1, i.e. ceil((P + W) C / T) (at most C). Both are
-// estimated in fp32 and then corrected against the table, which makes them exact.
-__device__ __forceinline__ void seg_cta_range(const long long* cuts, long long T, int C, long long P,
-                                              long long W, int& c0, int& c1) {
-  int c = (int)ceilf((float)(P + 1) * (float)C / (float)T) - 1;
-  c = max(0, min(C - 1, c));
-  while (c > 0 && cuts[c] > P) --c;
-  while (c < C - 1 && cuts[c + 1] <= P) ++c;
-  c0 = c;
-  const long long X = P + W - 1;
-  c = min((int)ceilf((float)(P + W) * (float)C / (float)T), C) - 1;
-  c = max(0, min(C - 1, c));
-  while (c < C - 1 && cuts[c + 1] <= X) ++c;
-  while (c > 0 && cuts[c] > X) --c;
-  c1 = c;
-}
-
-constexpr int kMaxCtas = 1024;   // grid size bound (64-bit cost-line arithmetic)
-static_assert(kMaxCtas < (1 << 16), "udiv_small divides by the grid size");
 
 // Completion counting (the first kDecodeCounterBytes of the workspace, DecodeHeader): a count of
 // the fused calls made on the workspace, and two sets of per-(sequence, KV head) arrival counters
@@ -672,7 +551,7 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
         if (issue_chunk(pr, sm, cK, cV, ring_w + ((n_issued + i) % ST) * STAGE,
                         &bars[(n_issued + i) % ST], total, lane, policy)) ++n_pending;
       int c0, c1;   // the CTAs that share this segment (their partials are merged by the last one)
-      seg_cta_range(cuts, T, C, P, W, c0, c1);
+      seg_cta_range([&](int i) { return cuts[i]; }, T, C, P, W, c0, c1);
       __syncwarp();
       rot_compute(sm, rr, s.grp, warp, lane);
       __syncthreads();
@@ -858,7 +737,7 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
           if (ok) { __syncwarp(); next_chunk(); }         // the last chunk of the item
         }
         cons_k += NW;
-        if (cons_k < total) cons = next_rr(sm, cons, cons_k);
+        if (cons_k < total) cons = next_rr<NW>(sm, cons, cons_k);
       }
       // drain: never leave bulk copies in flight into this ring (a copy whose wait gave up stays
       // counted in n_pending and is waited for once more before the CTA exits)

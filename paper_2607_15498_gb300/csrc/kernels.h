@@ -68,6 +68,17 @@ int launch_decode(const Shape& s, const varrate_packed& cache, const void* basis
                   const void* tail_v, int n_tail, void* out, int32_t* dev_status, void* ws,
                   int num_sms, cudaStream_t st);
 
+// ---- decode of a window of n_q new tokens, bf16 (decode_window.cu): q~ fragments, the coded part
+// on the cost line, then merge + causal exact tail + U_V^T per (sequence, KV head). The workspace
+// holds the q~ fragments and the per-(segment, CTA) partials, sized for kWindowMaxRows query rows.
+constexpr int kWindowMaxRows = 128;   // n_q * group
+size_t decode_window_ws_bytes(const Shape& s, int num_sms);
+bool decode_window_supported(const Shape& s, int n_q, int n_tail, int num_sms);
+int launch_decode_window(const Shape& s, const varrate_packed& c, const void* basis_k, const void* basis_v,
+                         const void* q, int n_q, int layer, const void* tail_k, const void* tail_v,
+                         int n_tail, void* out, int32_t* dev_status, void* ws, int num_sms,
+                         cudaStream_t st);
+
 // ---- quantized coefficients (quant.cu; decode with the general kernels in decode.cu)
 int launch_quantize(const Shape& s, const varrate_packed& in, const varrate_qpacked& out,
                     int32_t* dev_status, cudaStream_t st);

@@ -37,7 +37,7 @@ OK, FLOOR_BINDS = 0, 1
 ERR_ARG, ERR_WORKSPACE, ERR_CUDA, ERR_TIMEOUT, ERR_UNSUPPORTED, ERR_CORRUPT = -1, -2, -3, -4, -5, -6
 F32, BF16 = 0, 1
 SALIENCE, UNIFORM = 0, 1
-CALL_SALIENCE, CALL_PACK, CALL_ENCODE, CALL_DECODE = 0, 1, 2, 3
+CALL_SALIENCE, CALL_PACK, CALL_ENCODE, CALL_DECODE, CALL_DECODE_WINDOW = 0, 1, 2, 3, 4
 
 _c_void_p = ctypes.c_void_p
 
@@ -86,6 +86,11 @@ _SIGS = {
                                              _c_void_p, ctypes.c_int32, _c_void_p, _c_void_p,
                                              ctypes.c_int32, _c_void_p, _c_void_p, _c_void_p,
                                              ctypes.c_size_t, _c_void_p]),
+    "varrate_decode_window": (ctypes.c_int32, [ctypes.POINTER(varrate_config),
+                                               ctypes.POINTER(varrate_packed), _c_void_p, _c_void_p,
+                                               _c_void_p, ctypes.c_int32, ctypes.c_int32, _c_void_p,
+                                               _c_void_p, ctypes.c_int32, _c_void_p, _c_void_p,
+                                               _c_void_p, ctypes.c_size_t, _c_void_p]),
     "varrate_qpacked_cap_bytes": (ctypes.c_int64, [ctypes.POINTER(varrate_config), ctypes.c_int32]),
     "varrate_quantize": (ctypes.c_int32, [ctypes.POINTER(varrate_config), ctypes.POINTER(varrate_packed),
                                           ctypes.POINTER(varrate_qpacked), _c_void_p, _c_void_p]),
@@ -222,6 +227,14 @@ def varrate_decode_attn_noalloc(cfg, packed, basis_k, basis_v, q, layer, tail_k,
                                              _ptr(dev_status), _stream(stream))
 
 
+def varrate_decode_window(cfg, packed, basis_k, basis_v, q, n_q, layer, tail_k, tail_v, n_tail, out,
+                          dev_status, ws, stream=None) -> int:
+    return lib().varrate_decode_window(ctypes.byref(cfg), ctypes.byref(packed.c), _ptr(basis_k),
+                                       _ptr(basis_v), _ptr(q), n_q, layer, _ptr(tail_k), _ptr(tail_v),
+                                       n_tail, _ptr(out), _ptr(dev_status), _ptr(ws), _nbytes(ws),
+                                       _stream(stream))
+
+
 def varrate_qpacked_cap_bytes(cfg: varrate_config, bits: int) -> int:
     return lib().varrate_qpacked_cap_bytes(ctypes.byref(cfg), bits)
 
@@ -309,7 +322,7 @@ class QPackedCache:
 
 
 def workspace(cfg: varrate_config, which_call: int, device="cuda") -> torch.Tensor:
-    """Device scratch for one kind of call, zero-filled (decode needs its completion words zero
-    before the first call that uses them; every call leaves them finished for the next one)."""
+    """Device scratch for one kind of call, zero-filled (the decode workspace's header must be zero
+    before the first decode call that uses it; later calls keep it consistent themselves)."""
     n = varrate_workspace_bytes(cfg, which_call)
     return torch.zeros(max(n, 256), dtype=torch.uint8, device=device)

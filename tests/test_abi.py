@@ -142,6 +142,34 @@ def test_small_workspace_and_bad_layer_rejected_on_host(vlib):
                             None, A, 8, None) == vlib.ERR_WORKSPACE
 
 
+def test_window_decode_rejected_on_host(vlib):
+    """varrate_decode_window: bf16 only, 1 <= n_q <= n_tail, n_q * group <= 128, and a workspace of
+    varrate_workspace_bytes(cfg, VARRATE_CALL_DECODE_WINDOW), all checked before any launch."""
+    L = vlib.lib()
+    cfg = vlib.make_config(2, 2, 4, 2048, batch=2, dtype=vlib.BF16)
+    cap = vlib.varrate_packed_cap_elems(cfg)
+    p = vlib.varrate_packed(A, A, A, A, A, A, cap)
+    big = 1 << 40
+    need = vlib.varrate_workspace_bytes(cfg, vlib.CALL_DECODE_WINDOW)
+    assert need > 0 and need % 256 == 0
+
+    def call(c=cfg, n_q=4, layer=0, n_tail=8, tk=A, ws=A, nbytes=big, q=A):
+        return L.varrate_decode_window(vlib.ctypes.byref(c), vlib.ctypes.byref(p), A, A, q, n_q, layer,
+                                       tk, tk, n_tail, A, A, ws, nbytes, None)
+
+    assert call(tk=None) == vlib.ERR_ARG
+    assert call(n_q=0) == vlib.ERR_ARG
+    assert call(n_q=9, n_tail=8) == vlib.ERR_ARG
+    assert call(layer=2) == vlib.ERR_ARG
+    assert call(q=A + 2) == vlib.ERR_ARG
+    assert call(n_q=33, n_tail=40) == vlib.ERR_UNSUPPORTED      # 132 query rows
+    assert call(n_tail=5000) == vlib.ERR_UNSUPPORTED
+    assert call(nbytes=need - 256) == vlib.ERR_WORKSPACE
+    assert call(ws=None) == vlib.ERR_WORKSPACE
+    f32 = vlib.make_config(2, 2, 4, 2048, batch=2, dtype=vlib.F32)
+    assert call(c=f32) == vlib.ERR_UNSUPPORTED
+
+
 def test_misaligned_pointers_rejected_on_host(vlib):
     """Bulk copies and TMA need 16-byte aligned addresses: a misaligned device pointer is an
     argument error found on the host, before anything is enqueued."""
