@@ -23,6 +23,12 @@ constexpr float kSlack = 8.f;                // headroom of the running max, log
 // the combine), about as long as streaming this many coefficients at a CTA's share of HBM
 // bandwidth, so ranges that straddle segments are shortened by that much.
 constexpr long long kSegCost = 90112;
+// Cost-line allowance after each segment's coefficients: the CTA that takes a segment's last
+// stretch also pays its arrival, often the segment's combine, and the uneven finish of its warps on
+// the last items, so its range is shortened by this much. Both allowances were swept on the GPU
+// for the 32-layer, 8-sequence llama shape (64 segments over 152 CTAs); shapes with few segments
+// per grid barely feel them.
+constexpr long long kSegEnd = 163840;
 constexpr int kMaxCtas = 1024;   // grid size bound (64-bit cost-line arithmetic)
 
 // A 64-bit integer division is a long instruction sequence (measured ~600 cycles here), so the
@@ -143,7 +149,9 @@ __device__ __forceinline__ uint32_t keep_rows(uint32_t w, int j, int r) {
 
 // Per-sequence stream length segW[b] (equal for every head of the sequence; a table outside
 // [0, cap] counts as empty) and cost-line start segP[b] of sequence b, whose G segments take
-// kSegCost + segW[b] elements each (an empty sequence takes none); segP[64] = T, the line's length.
+// kSegCost + segW[b] + kSegEnd elements each (an empty sequence takes none); segP[64] = T, the
+// line's length. Segment (b, g)'s coefficients start at segP[b] + g (W_b + kSegCost + kSegEnd) +
+// kSegCost.
 // Called by every thread of the block (B <= 64, two sequences per lane of warp 0 in the scan);
 // ends with __syncthreads().
 __device__ __forceinline__ void seg_lengths(const int64_t* __restrict__ bucket_base, const Shape& s,
@@ -156,8 +164,8 @@ __device__ __forceinline__ void seg_lengths(const int64_t* __restrict__ bucket_b
   if (tid < 32) {
     const int lane = tid;
     const int e0 = 2 * lane, e1 = 2 * lane + 1;
-    const long long v0 = (e0 < s.B && segW[e0]) ? (segW[e0] + kSegCost) * s.G : 0;
-    const long long v1 = (e1 < s.B && segW[e1]) ? (segW[e1] + kSegCost) * s.G : 0;
+    const long long v0 = (e0 < s.B && segW[e0]) ? (segW[e0] + kSegCost + kSegEnd) * s.G : 0;
+    const long long v1 = (e1 < s.B && segW[e1]) ? (segW[e1] + kSegCost + kSegEnd) * s.G : 0;
     long long inc = v0 + v1;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
@@ -171,9 +179,10 @@ __device__ __forceinline__ void seg_lengths(const int64_t* __restrict__ bucket_b
   __syncthreads();
 }
 
-// The segment (b, g) whose span [segP[b] + g (W_b + kSegCost), ... + W_b + kSegCost) holds cost-line
-// position x (b = B when x lies past the line).
-__device__ __forceinline__ void segment_at(const long long* segP, const long long* segW, int B,
+// The first segment (b, g) whose coefficients end after cost-line position x: the segment whose
+// span [segP[b] + g (W_b + kSegCost + kSegEnd), ...) holds x, or the next one when x lies in that
+// span's end allowance (b = B when there is none).
+__device__ __forceinline__ void segment_at(const long long* segP, const long long* segW, int B, int G,
                                            long long x, int& b, int& g) {
   int lo_b = 0, hi_b = B;
   while (lo_b < hi_b) {
@@ -183,10 +192,17 @@ __device__ __forceinline__ void segment_at(const long long* segP, const long lon
   b = lo_b;
   g = 0;
   if (b < B) {   // g = floor(y / w), estimated in fp32 and corrected
-    const long long y = x - segP[b], w = segW[b] + kSegCost;
+    const long long y = x - segP[b], w = segW[b] + kSegCost + kSegEnd;
     g = (int)((float)y / (float)w);
     while (g > 0 && (long long)g * w > y) --g;
     while ((long long)(g + 1) * w <= y) ++g;
+    if (y - (long long)g * w >= kSegCost + segW[b]) {   // in the end allowance: the next segment
+      if (++g == G) {
+        g = 0;
+        ++b;
+        while (b < B && segW[b] == 0) ++b;
+      }
+    }
   }
 }
 

@@ -12,9 +12,9 @@
 // is read as K chunks then V chunks of up to 8 KB each (32 rows of a full tile, 64 or 128 rows of a
 // short one), each one contiguous block.
 //
-// Memory path. Each warp owns a 3-stage shared-memory ring filled by one 1-D TMA bulk copy per
-// chunk that completes on a per-stage mbarrier; while the warp computes on one stage the other
-// two are in flight (the stage it finishes is refilled with the chunk three ahead), across item
+// Memory path. Each of the 12 warps owns a 2-stage shared-memory ring filled by one 1-D TMA bulk
+// copy per chunk that completes on a per-stage mbarrier; while the warp computes on one stage the
+// other is in flight (the stage it finishes is refilled with the chunk two ahead), across item
 // boundaries, so loads never wait on arithmetic. The per-row rotation of
 // the 8-slot groups keeps the unpadded staged rows free of shared-memory bank conflicts. Rows >= r
 // of a chunk are never loaded: they are masked out of the K and V fragments (not multiplied by
@@ -46,8 +46,11 @@ namespace vr {
 
 namespace {
 
-constexpr int NW = 8;                 // warps per CTA
-constexpr int ST = 3;                 // ring stages per warp
+// 12 warps of at most 168 registers fill the register file, three per scheduler: more warps hide
+// more of the instruction latency of the item loop than deeper rings do (measured: 8 warps with 3
+// stages each 54.7 us per llama32 layer call, 12 warps with 2 stages 52.2 us, same 192 KB ring).
+constexpr int NW = 12;                // warps per CTA
+constexpr int ST = 2;                 // ring stages per warp
 constexpr int kPartStride = kHeadDim + 4;   // o~[128], max, sum, pad: rows 16-byte aligned
 constexpr int kHeadsPad = 8;
 
@@ -115,7 +118,7 @@ __device__ __forceinline__ bool issue_chunk(Prod& p, const SegSmem& sm, const __
 // warp w computing rows j in [16w, 16w + 16) with one m16n8k16 tile per 16 columns of U_K. The
 // loads (rot_load) are issued at the start of a segment, ahead of its table loads, so both take
 // one memory round trip together; rot_compute runs once the tables are in.
-static_assert(NW * 16 == kHeadDim, "one 16-row tile of U_K per warp");
+static_assert(NW * 16 >= kHeadDim, "one 16-row tile of U_K per warp (warps past d / 16 idle)");
 struct RotRegs {
   uint32_t a[kHeadDim / 16][4];    // U_K rows 16w .. 16w + 15 (A fragments)
   uint32_t bq[kHeadDim / 16][2];   // q (B fragments; zero for padded heads)
@@ -206,10 +209,10 @@ struct CombSmem {   // aliases the ring while the last CTA of a segment combines
   float hl[kHeadsPad];                                      // softmax normaliser per head
 };
 static_assert(sizeof(CombSmem) <= (size_t)NW * ST * STAGE, "combine buffers fit in the ring");
-static_assert(NW == kHeadsPad, "one warp per head in the combine");
+static_assert(NW >= kHeadsPad, "one warp per head in the combine");
 
 // Merge the partials of segment (b, g) written by CTAs c0..c1 (slot cc + seg; none if c1 < c0),
-// add the exact tail, rotate back with U_V^T and normalise. Called by all 256 threads; the ring
+// add the exact tail, rotate back with U_V^T and normalise. Called by all threads; the ring
 // is idle. U_V and the tail's keys and values are staged in the ring by bulk copies while the
 // partials are merged (warp h merges head h, lane l columns 4l .. 4l + 3, with the partials of up
 // to 8 CTAs in flight at once). Tail scores are m16n8k16 tiles (16 tail tokens x 8 heads, exact
@@ -289,7 +292,7 @@ __device__ bool combine_segment(CombSmem& cs, uint64_t* bar, uint32_t parity, co
   }
   if (!__syncthreads_and(mbar_wait_bounded(bar, parity, kWaitTries))) return false;
   __syncwarp();
-  // exact tail scores (log2 units): warp w takes tail tiles w, w + 8, ...
+  // exact tail scores (log2 units): warp w takes tail tiles w, w + NW, ...
   const float scale = kLog2e * rsqrtf((float)kHeadDim);
   for (int tt = warp; tt < n_tt; tt += NW) {
     float sc[4] = {0.f, 0.f, 0.f, 0.f};
@@ -320,18 +323,18 @@ __device__ bool combine_segment(CombSmem& cs, uint64_t* bar, uint32_t parity, co
     float lt = 0.f;
     for (int t = lane; t < n_tt * 16; t += 32) {
       const float w = (h < grp && t < n_tail) ? exp2f(cs.tsc[h][t] - mx) : 0.f;
-      cs.tsc[h][t] = w;   // zero for padded heads and rows past the tail
+      if (h < kHeadsPad) cs.tsc[h][t] = w;   // zero for padded heads and rows past the tail
       lt += w;
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) lt += __shfl_xor_sync(0xffffffffu, lt, o);
-    if (lane == 0) cs.hl[h] = L * f + lt;
+    if (lane == 0 && h < kHeadsPad) cs.hl[h] = L * f + lt;
     if (h >= grp) acc = make_float4(0.f, 0.f, 0.f, 0.f);
-    *reinterpret_cast<float4*>(&cs.ot[h][4 * lane]) = acc;     // zero for padded heads
+    if (h < kHeadsPad) *reinterpret_cast<float4*>(&cs.ot[h][4 * lane]) = acc;   // zero for padded heads
   }
   __syncthreads();
-  // out^T[col][head]: warp w owns columns 16w .. 16w + 15
-  {
+  // out^T[col][head]: warp w < 8 owns columns 16w .. 16w + 15
+  if (warp < kHeadDim / 16) {
     // four independent accumulators (hi / lo part of the B operand, even / odd k-step) keep the
     // chain of dependent MMAs short
     float d[4][4] = {};
@@ -436,13 +439,13 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
   // the other CTAs stay consistent.
   bool dead = false;
   uint32_t n_comb = 0;     // combines done by this CTA (phase of bar_comb)
-  // Cost line: sequence b holds G segments of kSegCost + W_b elements each (W_b > 0), the set-up
-  // allowance first. segP = exclusive prefix over sequences (B <= 64: two per lane).
+  // Cost line: sequence b holds G segments of kSegCost + W_b + kSegEnd elements each (W_b > 0): the
+  // set-up allowance, the coefficients, the end allowance. segP = exclusive prefix over sequences (B <= 64: two per lane).
   if (warp == 0) {
     __syncwarp();   // lanes left the loads above apart: reconverge before the shuffles
     const int e0 = 2 * lane, e1 = 2 * lane + 1;
-    const long long v0 = (e0 < s.B && segW[e0]) ? (segW[e0] + kSegCost) * s.G : 0;
-    const long long v1 = (e1 < s.B && segW[e1]) ? (segW[e1] + kSegCost) * s.G : 0;
+    const long long v0 = (e0 < s.B && segW[e0]) ? (segW[e0] + kSegCost + kSegEnd) * s.G : 0;
+    const long long v1 = (e1 < s.B && segW[e1]) ? (segW[e1] + kSegCost + kSegEnd) * s.G : 0;
     long long inc = v0 + v1;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
@@ -472,13 +475,17 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
     }
     b = lo_b;
     if (b < s.B) {   // g = floor(x / w), estimated in fp32 and corrected
-      const long long x = lo_g - segP[b], w = segW[b] + kSegCost;
+      const long long x = lo_g - segP[b], w = segW[b] + kSegCost + kSegEnd;
       g = (int)((float)x / (float)w);
       while (g > 0 && (long long)g * w > x) --g;
       while ((long long)(g + 1) * w <= x) ++g;
     }
   }
-  auto seg_start = [&](int bb, int gg) { return segP[bb] + gg * (segW[bb] + kSegCost) + kSegCost; };
+  auto seg_start = [&](int bb, int gg) { return segP[bb] + gg * (segW[bb] + kSegCost + kSegEnd) + kSegCost; };
+  if (b < s.B && seg_start(b, g) + segW[b] <= lo_g) {   // the range starts in a segment's end allowance
+    if (++g == s.G) { ++b; g = 0; }
+    while (b < s.B && segW[b] == 0) ++b;
+  }
   bool more = b < s.B && seg_start(b, g) < hi_g;
   while (more) {
     {
@@ -553,7 +560,7 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
       int c0, c1;   // the CTAs that share this segment (their partials are merged by the last one)
       seg_cta_range([&](int i) { return cuts[i]; }, T, C, P, W, c0, c1);
       __syncwarp();
-      rot_compute(sm, rr, s.grp, warp, lane);
+      if (warp < kHeadDim / 16) rot_compute(sm, rr, s.grp, warp, lane);
       __syncthreads();
       build_qfrag(sm, tid);
       __syncthreads();
@@ -595,7 +602,6 @@ decode_mma_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restr
           const uint32_t st_addr = ring_w + (n_issued % ST) * STAGE;
           const int m = lane >> 3, r8 = lane & 7;
           const int j0 = jc << lgc, j1 = min(r, j0 + (1 << lgc));
-#pragma unroll 2
           for (int j16 = j0; j16 < j1; j16 += 16) {
             const uint4 qf = *reinterpret_cast<const uint4*>(&sm.qfrag[j16 >> 4][lane][0]);
             // this lane's row of the 8x8 matrices: coefficient j, staged at row (j - chunk start)
@@ -879,7 +885,7 @@ size_t decode_mma_part_bytes(const Shape& s, int num_sms) {
 
 bool decode_mma_supported(const Shape& s, int n_tail, int num_sms) {
   // the cost line (at most B G cap elements) times the grid size must stay below 2^62
-  const unsigned long long line = (unsigned long long)s.B * s.G * ((unsigned long long)s.cap + kSegCost);
+  const unsigned long long line = (unsigned long long)s.B * s.G * ((unsigned long long)s.cap + kSegCost + kSegEnd);
   return s.dtype == VARRATE_BF16 && s.B <= 64 && (long long)s.B * s.G <= kDecodeMaxSegs &&
          n_tail <= kMaxTailFused && num_sms >= 1 && num_sms <= kMaxCtas &&
          line <= (1ull << 62) / (unsigned long long)num_sms;

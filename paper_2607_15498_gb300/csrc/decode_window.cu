@@ -224,8 +224,8 @@ decode_window_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __re
   __syncthreads();
   const long long lo_g = cuts[cta], hi_g = cuts[cta + 1];
   int b, g;
-  segment_at(segP, segW, s.B, lo_g, b, g);
-  auto seg_start = [&](int bb, int gg) { return segP[bb] + gg * (segW[bb] + kSegCost) + kSegCost; };
+  segment_at(segP, segW, s.B, s.G, lo_g, b, g);
+  auto seg_start = [&](int bb, int gg) { return segP[bb] + gg * (segW[bb] + kSegCost + kSegEnd) + kSegCost; };
   bool more = b < s.B && seg_start(b, g) < hi_g;
 
   const uint32_t ring_t = ring + team * SPT * STAGE;
@@ -655,7 +655,7 @@ window_combine_kernel(const float* __restrict__ part, const int64_t* __restrict_
   const long long W = segW[b];
   if (W > 0 && valid) {
     const long long T = segP[64];
-    const long long P = segP[b] + g * (W + kSegCost) + kSegCost;
+    const long long P = segP[b] + g * (W + kSegCost + kSegEnd) + kSegCost;
     int c0, c1;
     seg_cta_range([&](int i) { return cut_at(T, i, C); }, T, C, P, W, c0, c1);
     for (int p = c0; p <= c1; ++p) {
@@ -810,7 +810,7 @@ size_t decode_window_ws_bytes(const Shape& s, int num_sms) {
 }
 
 bool decode_window_supported(const Shape& s, int n_q, int n_tail, int num_sms) {
-  const unsigned long long line = (unsigned long long)s.B * s.G * ((unsigned long long)s.cap + kSegCost);
+  const unsigned long long line = (unsigned long long)s.B * s.G * ((unsigned long long)s.cap + kSegCost + kSegEnd);
   return s.dtype == VARRATE_BF16 && s.B <= 64 && n_q >= 1 && n_q <= n_tail &&
          (long long)n_q * s.grp <= kWindowMaxRows && (long long)s.B * s.G < (1LL << 31) &&
          num_sms >= 1 && num_sms <= kMaxCtas && line <= (1ull << 62) / (unsigned long long)num_sms;
