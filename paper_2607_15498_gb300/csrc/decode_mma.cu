@@ -131,7 +131,8 @@ struct RotRegs {
 // fragment register a0 (t % 4 < 2) or a2 (t % 4 >= 2).
 __device__ __forceinline__ void rot_load(RotRegs& rr, const __nv_bfloat16* __restrict__ U,
                                          const __nv_bfloat16* __restrict__ q, int grp, int warp, int lane) {
-  const int g8 = lane >> 2, c = lane & 3, j0 = warp * 16;
+  // warps past d / 16 load (and never use) the tile of warp w mod 8: every address stays in U
+  const int g8 = lane >> 2, c = lane & 3, j0 = (warp % (kHeadDim / 16)) * 16;
   const uint4* u0 = reinterpret_cast<const uint4*>(U + (long long)(j0 + g8) * kHeadDim) + c;
   const uint4* u1 = reinterpret_cast<const uint4*>(U + (long long)(j0 + g8 + 8) * kHeadDim) + c;
   const uint4* qr = reinterpret_cast<const uint4*>(q + (long long)(g8 < grp ? g8 : 0) * kHeadDim) + c;
