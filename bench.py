@@ -69,10 +69,10 @@ def measured_traffic():
 
 
 def kernel_source_sha256():
-    """sha256 over the decode kernel's sources (decode_mma.cu, then common.cuh)."""
+    """sha256 over the decode kernel's sources (decode_mma.cu, decode_common.cuh, common.cuh)."""
     import hashlib
     h = hashlib.sha256()
-    for name in ("decode_mma.cu", "common.cuh"):
+    for name in ("decode_mma.cu", "decode_common.cuh", "common.cuh"):
         h.update(open(os.path.join(ROOT, "paper_2607_15498_gb300", "csrc", name), "rb").read())
     return h.hexdigest()
 
