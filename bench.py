@@ -268,25 +268,27 @@ def run_e2e(args, V, cfg, wl, k, v, qw, bk, bv, qdec, packed, realized, status, 
     hq.copy_(qw)
     hqd.copy_(qdec)
     dk, dv, dq = torch.empty_like(k), torch.empty_like(v), torch.empty_like(qw)
-    dqs = torch.empty_like(qdec[0, 0])
-    dout = torch.empty((cfg.batch, wl.n_q_heads, wl.head_dim), dtype=k.dtype, device=k.device)
+    dqd = torch.empty_like(qdec)
+    # one output slot per (decode step, layer): the step's results leave in one read at its end
+    dout = torch.empty((D, L, cfg.batch, wl.n_q_heads, wl.head_dim), dtype=k.dtype, device=k.device)
     hout = torch.empty(dout.shape, dtype=dout.dtype, pin_memory=True)
     torch.cuda.synchronize()
 
     def one_step(evs):
+        # the step's inputs (K, V, window queries, every decode query) in from pinned host memory
         evs[0].record(stream)
         dk.copy_(hk, non_blocking=True)
         dv.copy_(hv, non_blocking=True)
         dq.copy_(hq, non_blocking=True)
+        dqd.copy_(hqd, non_blocking=True)
         V.check(V.varrate_encode(cfg, dq, dk, dv, bk, bv, None, packed, realized, status, ws_enc,
                                  stream))
         evs[1].record(stream)
         for s in range(D):
             for l in range(L):
-                dqs.copy_(hqd[s, l], non_blocking=True)
-                V.check(V.varrate_decode_attn(cfg, packed, bk, bv, dqs, l, None, None, 0, dout,
-                                              status, ws_dec, stream))
-                hout.copy_(dout, non_blocking=True)
+                V.check(V.varrate_decode_attn(cfg, packed, bk, bv, dqd[s, l], l, None, None, 0,
+                                              dout[s, l], status, ws_dec, stream))
+        hout.copy_(dout, non_blocking=True)   # every output of the step back to the host
         evs[2].record(stream)
 
     one_step([torch.cuda.Event(enable_timing=True) for _ in range(3)])   # warm
@@ -299,7 +301,7 @@ def run_e2e(args, V, cfg, wl, k, v, qw, bk, bv, qdec, packed, realized, status, 
         enc.append(evs[0].elapsed_time(evs[1]))
         dec.append(evs[1].elapsed_time(evs[2]))
     h2d = (hk.numel() + hv.numel() + hq.numel() + hqd.numel()) * hk.element_size()
-    d2h = D * L * hout.numel() * hout.element_size()
+    d2h = hout.numel() * hout.element_size()
     dec_gbs = D * sum(dec_bytes) / (statistics.mean(dec) * 1e-3) / 1e9
     return {"value": round(dec_gbs, 1), "unit": "GB/s",
             "encode_ms_per_32k_ctx": round(statistics.mean(enc) / cfg.batch, 3),
