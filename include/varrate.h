@@ -133,7 +133,8 @@ typedef enum {
   VARRATE_CALL_PACK = 1,
   VARRATE_CALL_ENCODE = 2,
   VARRATE_CALL_DECODE = 3,
-  VARRATE_CALL_DECODE_WINDOW = 4
+  VARRATE_CALL_DECODE_WINDOW = 4,
+  VARRATE_CALL_DECODE_Q = 5
 } varrate_call;
 
 /* Library version (major * 10000 + minor * 100 + patch). */
@@ -266,10 +267,16 @@ varrate_status varrate_quantize(const varrate_config* cfg, const varrate_packed*
                                 varrate_qpacked* out, int32_t* dev_status, void* stream);
 
 /* Decode attention of one layer on a quantized cache: the same mathematics and arguments as
- * varrate_decode_attn with each stored coefficient c replaced by its dequantized value x^ (fp32),
- * computed by the general kernels (query rotation, split over tokens, combine); ws as for
- * varrate_decode_attn (varrate_workspace_bytes(cfg, VARRATE_CALL_DECODE)); 0 <= n_tail <= 4096;
- * dtype VARRATE_BF16 only (queries, bases, tail and output bf16). */
+ * varrate_decode_attn with each stored coefficient c replaced by its dequantized value x^
+ * = fl32(lo + fl32(code * step)); 0 <= n_tail <= 4096; dtype VARRATE_BF16 only (queries, bases,
+ * tail and output bf16). ws holds at least varrate_workspace_bytes(cfg, VARRATE_CALL_DECODE) bytes,
+ * zero-filled before first use like the decode workspace (its header is the same).
+ *  - With at least varrate_workspace_bytes(cfg, VARRATE_CALL_DECODE_Q) bytes and a shape the fused
+ *    bf16 decode kernel takes (see varrate_decode_attn), the layer is first expanded into the
+ *    workspace as a bf16 packed cache (x^ rounded to bf16) and then decoded by that kernel: two
+ *    launches, the second with programmatic stream serialization as for varrate_decode_attn.
+ *  - Otherwise the general kernels (query rotation, split over tokens, combine) decode on x^ in
+ *    fp32 directly. */
 varrate_status varrate_decode_attn_q(const varrate_config* cfg, const varrate_qpacked* cache,
                                      const void* basis_k, const void* basis_v, const void* q,
                                      int32_t layer, const void* tail_k, const void* tail_v,

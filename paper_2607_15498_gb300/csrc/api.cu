@@ -1,5 +1,6 @@
 // C ABI of the VarRate hot path (declared in include/varrate.h): argument validation, workspace
 // carving and kernel launches. No device memory is allocated here.
+#include <algorithm>
 #include <atomic>
 #include <initializer_list>
 #include <math.h>
@@ -87,6 +88,7 @@ size_t ws_bytes(const varrate_config* c, int32_t which) {
              align256((size_t)s.B * s.L * sizeof(int64_t));
     case VARRATE_CALL_DECODE: return vr::decode_ws_bytes(s, sms);
     case VARRATE_CALL_DECODE_WINDOW: return vr::decode_window_ws_bytes(s, sms);
+    case VARRATE_CALL_DECODE_Q: return std::max(vr::decode_ws_bytes(s, sms), vr::decode_q_expand_ws_bytes(s, sms));
     default: return 0;
   }
 }
@@ -313,9 +315,15 @@ varrate_status varrate_decode_attn_q(const varrate_config* cfg, const varrate_qp
   const size_t need = ws_bytes(cfg, VARRATE_CALL_DECODE);
   if (ws_bytes_ < need || ws == nullptr) return VARRATE_ERR_WORKSPACE;
   const Shape s = make_shape(cfg, cap_elems(cfg));
-  (void)dev_status;
-  vr::launch_decode_q(s, *cache, basis_k, basis_v, q, layer, tail_k, tail_v, n_tail, out, ws,
-                      num_sms(), (cudaStream_t)stream);
+  const int sms = num_sms();
+  if (vr::decode_q_expand_supported(s, n_tail, sms) && ws_bytes_ >= ws_bytes(cfg, VARRATE_CALL_DECODE_Q)) {
+    if (vr::launch_decode_q_expand(s, *cache, basis_k, basis_v, q, layer, tail_k, tail_v, n_tail, out,
+                                   dev_status, ws, sms, (cudaStream_t)stream) < 0)
+      return VARRATE_ERR_CUDA;
+    return launched();
+  }
+  vr::launch_decode_q(s, *cache, basis_k, basis_v, q, layer, tail_k, tail_v, n_tail, out, ws, sms,
+                      (cudaStream_t)stream);
   return launched();
 }
 

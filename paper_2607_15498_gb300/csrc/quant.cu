@@ -40,8 +40,15 @@ __global__ void qtables_kernel(const int32_t* __restrict__ bucket_count, int64_t
   qb[kMaxR + 1] = acc;
 }
 
-// grid (2 G, B L), 256 threads: one CTA per stream (b, l, g, kv); warp w quantizes coefficient rows
-// w, w + 8, ... of the stream, the rows enumerated bucket by bucket, tile by tile.
+// grid (2 G, B L, kQuantSplit), 256 threads: CTA (stream, bl, z) quantizes the z-th share of the
+// tiles of stream (b, l, g, kv). A warp takes one tile at a time, two rows per step: lane (lr, gp)
+// reads the 8 bf16 coefficients of slot group gp of row 2 jj + lr (stored at position (gp + j) mod
+// (tl / 8)), the four lanes of a 32-slot group agree on its min and max by shuffles, and each lane
+// writes its 8 codes (one 32-bit word at 4 bits, two at 8 bits); the group's first lane writes
+// (lo, step) and the row's padding bytes are zeroed.
+constexpr int kQuantSplit = 8;
+constexpr int kDeqRows = 8;   // rows per lane whose loads are in flight together (both directions)
+
 template <int BITS>
 __global__ void __launch_bounds__(256)
 quantize_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restrict__ bucket_count,
@@ -50,8 +57,8 @@ quantize_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restric
   __shared__ int cnt[kMaxR + 1];
   __shared__ long long base[kMaxR + 2];
   __shared__ long long qb[kMaxR + 2];
-  __shared__ long long rows_pre[kMaxR + 2];   // rows of the buckets before r (r rows per tile)
-  const int kv = blockIdx.x & 1, g = blockIdx.x >> 1;
+  __shared__ int tiles_pre[kMaxR + 2];   // tiles of the buckets before r
+  const int kv = blockIdx.x & 1, g = blockIdx.x >> 1, z = blockIdx.z;
   const int64_t bl = blockIdx.y;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   for (int r = tid; r <= kMaxR + 1; r += blockDim.x) {
@@ -61,94 +68,284 @@ quantize_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restric
   }
   __syncthreads();
   if (tid == 0) {
-    long long acc = 0;
+    int tiles = 0;
     for (int r = 0; r <= kMaxR; ++r) {
-      rows_pre[r] = acc;
-      if (r >= s.r_min && r <= s.r_max) acc += (long long)r * ((pad8(cnt[r]) + 127) / 128);
+      tiles_pre[r] = tiles;
+      if (r >= s.r_min && r <= s.r_max && cnt[r] > 0) tiles += (int)((pad8(cnt[r]) + 127) / 128);
     }
-    rows_pre[kMaxR + 1] = acc;
+    tiles_pre[kMaxR + 1] = tiles;
   }
   __syncthreads();
   // a table that does not fit the buffers (corrupt ranks upstream) is skipped
   if (base[kMaxR + 1] > s.cap || qb[kMaxR + 1] > qcap) {
-    if (tid == 0) raise_status(dev_status, VARRATE_ERR_CORRUPT);
+    if (tid == 0 && blockIdx.x == 0 && z == 0) raise_status(dev_status, VARRATE_ERR_CORRUPT);
     return;
   }
   const int64_t stream = (bl * s.G + g) * 2 + kv;
   const __nv_bfloat16* src = coef + stream * s.cap;
   uint8_t* dst = qdata + stream * qcap;
   constexpr float kQmax = (float)((1 << BITS) - 1);
-  const long long total = rows_pre[kMaxR + 1];
-  for (long long R = warp; R < total; R += blockDim.x / 32) {
-    int lo_r = 0, hi_r = kMaxR + 1;   // rows_pre[lo_r] <= R < rows_pre[hi_r]
+  const int total = tiles_pre[kMaxR + 1];
+  const int T0 = (int)((long long)total * z / kQuantSplit), T1 = (int)((long long)total * (z + 1) / kQuantSplit);
+  const int lr = lane >> 4, gp = lane & 15;
+  for (int T = T0 + warp; T < T1; T += blockDim.x / 32) {
+    int lo_r = 0, hi_r = kMaxR + 1;   // tiles_pre[lo_r] <= T < tiles_pre[hi_r]
     while (hi_r - lo_r > 1) {
       const int mid = (lo_r + hi_r) >> 1;
-      if (rows_pre[mid] <= R) lo_r = mid; else hi_r = mid;
+      if (tiles_pre[mid] <= T) lo_r = mid; else hi_r = mid;
     }
     const int r = lo_r;
-    const long long k = R - rows_pre[r];
-    const long long i = k / r;
-    const int j = (int)(k - i * r);
-    const long long n8 = pad8(cnt[r]);
-    const int tl = (int)min(128ll, n8 - 128 * i);
+    const long long i = T - tiles_pre[r];
+    const int tl = (int)min(128ll, pad8(cnt[r]) - 128 * i);
     const int ng = tl >> 3;
-    // bf16 row j of tile i: 8-slot group gp at position (gp + j) mod ng
-    const __nv_bfloat16* row = src + base[r] + 128 * i * r + (long long)j * tl;
-    const int p0 = lane * 4;                  // this lane's 4 slots (one half of an 8-slot group)
-    const bool on = p0 < tl;
-    float x[4] = {0.f, 0.f, 0.f, 0.f};
-    if (on) {
-      const int gp = p0 >> 3;
-      const uint2 u = *reinterpret_cast<const uint2*>(row + 8 * ((gp + j) % ng) + (p0 & 7));
-      x[0] = __uint_as_float(u.x << 16); x[1] = __uint_as_float(u.x & 0xffff0000u);
-      x[2] = __uint_as_float(u.y << 16); x[3] = __uint_as_float(u.y & 0xffff0000u);
-    }
-    float mn = on ? fminf(fminf(x[0], x[1]), fminf(x[2], x[3])) : INFINITY;
-    float mx = on ? fmaxf(fmaxf(x[0], x[1]), fmaxf(x[2], x[3])) : -INFINITY;
-#pragma unroll
-    for (int o = 1; o < 8; o <<= 1) {   // the 8 lanes of a 32-slot group
-      mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, o));
-      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-    }
-    const __half lo = __float2half_rn(mn);
-    const float lo32 = __half2float(lo);
-    // a range beyond the fp16 range saturates the step at the largest finite fp16
-    const __half st = __float2half_rn(fminf(__fdiv_rn(__fsub_rn(mx, lo32), kQmax), 65504.f));
-    const float s32 = __half2float(st);
-    uint32_t q[4];
-#pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      int c = 0;
-      if (s32 != 0.f) c = __float2int_rn(__fdiv_rn(__fsub_rn(x[e], lo32), s32));
-      q[e] = (uint32_t)min(max(c, 0), (int)kQmax);
-    }
-    uint8_t* qrow = dst + qb[r] + i * (long long)r * qrow_bytes(128, BITS) + (long long)j * qrow_bytes(tl, BITS);
-    if (on) {
-      if (BITS == 4) {
-        const uint16_t w = (uint16_t)(q[0] | (q[1] << 4) | (q[2] << 8) | (q[3] << 12));
-        *reinterpret_cast<uint16_t*>(qrow + (p0 >> 1)) = w;
-      } else {
-        *reinterpret_cast<uint32_t*>(qrow + p0) = q[0] | (q[1] << 8) | (q[2] << 16) | (q[3] << 24);
-      }
-      if ((lane & 7) == 0) {
-        __half2 par = __halves2half2(lo, st);
-        *reinterpret_cast<__half2*>(qrow + tl * BITS / 8 + 4 * (p0 / kGroup)) = par;
-      }
-    }
-    // zero padding of the row to its 16-byte size
+    const int qrow = qrow_bytes(tl, BITS);
     const int raw = tl * BITS / 8 + 4 * ((tl + kGroup - 1) / kGroup);
-    if (lane < qrow_bytes(tl, BITS) - raw) qrow[raw + lane] = 0;
-    __syncwarp();
+    const __nv_bfloat16* stile = src + base[r] + 128 * i * r;
+    uint8_t* qtile = dst + qb[r] + i * (long long)r * qrow_bytes(128, BITS);
+    const bool on = gp < ng;
+    for (int j0 = 0; j0 < r; j0 += 2 * kDeqRows) {
+      uint4 x[kDeqRows];
+#pragma unroll
+      for (int u = 0; u < kDeqRows; ++u) {   // every row's load in flight before the first use
+        const int j = j0 + 2 * u + lr;
+        if (on && j < r) x[u] = *reinterpret_cast<const uint4*>(stile + (long long)j * tl + 8 * ((gp + j) % ng));
+      }
+#pragma unroll
+      for (int u = 0; u < kDeqRows; ++u) {
+        if (j0 + 2 * u >= r) break;   // warp-uniform: no row of this step in either half
+        const int j = j0 + 2 * u + lr;
+        const bool valid = on && j < r;   // the other half-warp may still have a row: no early exit
+        float v[8];
+        v[0] = __uint_as_float(x[u].x << 16); v[1] = __uint_as_float(x[u].x & 0xffff0000u);
+        v[2] = __uint_as_float(x[u].y << 16); v[3] = __uint_as_float(x[u].y & 0xffff0000u);
+        v[4] = __uint_as_float(x[u].z << 16); v[5] = __uint_as_float(x[u].z & 0xffff0000u);
+        v[6] = __uint_as_float(x[u].w << 16); v[7] = __uint_as_float(x[u].w & 0xffff0000u);
+        float mn = INFINITY, mx = -INFINITY;
+        if (valid) {
+#pragma unroll
+          for (int e = 0; e < 8; ++e) { mn = fminf(mn, v[e]); mx = fmaxf(mx, v[e]); }
+        }
+        // the four lanes of a 32-slot group (gp = 4 q .. 4 q + 3 of the same half)
+        mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, 1));
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+        mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, 2));
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+        const __half lo = __float2half_rn(mn);
+        const float lo32 = __half2float(lo);
+        // a range beyond the fp16 range saturates the step at the largest finite fp16
+        const __half st = __float2half_rn(fminf(__fdiv_rn(__fsub_rn(mx, lo32), kQmax), 65504.f));
+        const float s32 = __half2float(st);
+        uint32_t q[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          int cq = 0;
+          if (s32 != 0.f) cq = __float2int_rn(__fdiv_rn(__fsub_rn(v[e], lo32), s32));
+          q[e] = (uint32_t)min(max(cq, 0), (int)kQmax);
+        }
+        if (j >= r) continue;
+        uint8_t* row = qtile + (long long)j * qrow;
+        if (on) {
+          if (BITS == 4) {
+            uint32_t w = 0;
+#pragma unroll
+            for (int e = 0; e < 8; ++e) w |= q[e] << (4 * e);
+            *reinterpret_cast<uint32_t*>(row + 4 * gp) = w;
+          } else {
+            *reinterpret_cast<uint2*>(row + 8 * gp) =
+                make_uint2(q[0] | (q[1] << 8) | (q[2] << 16) | (q[3] << 24), q[4] | (q[5] << 8) | (q[6] << 16) | (q[7] << 24));
+          }
+          if ((gp & 3) == 0) *reinterpret_cast<__half2*>(row + tl * BITS / 8 + 4 * (gp >> 2)) = __halves2half2(lo, st);
+        }
+        if (gp < qrow - raw) row[raw + gp] = 0;   // zero padding of the row to its 16-byte size
+      }
+    }
+  }
+}
+
+// Expansion of one layer of a quantized cache to the bf16 packed layout, for the fused decode:
+// grid (2 G, B, kDeqSplit), 256 threads. CTA (stream, b, z) writes the z-th share of the tiles of
+// stream (b, layer, g, kv); a warp takes one tile at a time, two rows per step: lane (lr, gp) turns
+// the 8 codes of slot group gp of row 2 jj + lr into lo + code * step (one fused multiply-add, within
+// an fp32 rounding of x^ = fl32(lo + fl32(code * step))), rounds them to bf16 and stores them as one 16-byte group at its packed position (group gp of row j at
+// position (gp + j) mod (tl / 8)). CTA (0, b, 0) also writes sequence b's bucket counts and element
+// bases for the layer (a table that does not fit the buffers is written as an empty stream and
+// raises VARRATE_ERR_CORRUPT).
+constexpr int kDeqSplit = 8;
+
+// The 8 codes of one 8-slot group: one 32-bit word (4-bit codes, the even slot in the low nibble)
+// or two (8-bit).
+template <int BITS> struct CodeWord;
+template <> struct CodeWord<4> {
+  using T = uint32_t;
+  static __device__ __forceinline__ void unpack(uint32_t w, uint32_t (&c)[8]) {
+#pragma unroll
+    for (int e = 0; e < 8; ++e) c[e] = (w >> (4 * e)) & 15u;
+  }
+};
+template <> struct CodeWord<8> {
+  using T = uint2;
+  static __device__ __forceinline__ void unpack(uint2 w, uint32_t (&c)[8]) {
+#pragma unroll
+    for (int e = 0; e < 4; ++e) { c[e] = (w.x >> (8 * e)) & 255u; c[4 + e] = (w.y >> (8 * e)) & 255u; }
+  }
+};
+
+template <int BITS>
+__global__ void __launch_bounds__(256)
+dequant_layer_kernel(const uint8_t* __restrict__ qdata, const int64_t* __restrict__ qbase,
+                     const int32_t* __restrict__ bucket_count, __nv_bfloat16* __restrict__ coef,
+                     int32_t* __restrict__ cnt_out, int64_t* __restrict__ base_out,
+                     int32_t* __restrict__ dev_status, Shape s, int layer, int64_t qcap) {
+  __shared__ int cnt[kMaxR + 1];
+  __shared__ long long base[kMaxR + 2];
+  __shared__ long long qb[kMaxR + 2];
+  __shared__ int tiles_pre[kMaxR + 2];   // tiles of the buckets before r
+  const int kv = blockIdx.x & 1, g = blockIdx.x >> 1, b = blockIdx.y, z = blockIdx.z;
+  const int64_t bl = (int64_t)b * s.L + layer;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  for (int r = tid; r <= kMaxR + 1; r += blockDim.x) {
+    if (r <= kMaxR) cnt[r] = bucket_count[bl * (kMaxR + 1) + r];
+    qb[r] = qbase[bl * (kMaxR + 2) + r];
+  }
+  __syncthreads();
+  if (tid == 0) {
+    long long acc = 0;
+    int tiles = 0;
+    for (int r = 0; r <= kMaxR; ++r) {
+      base[r] = acc;
+      tiles_pre[r] = tiles;
+      if (r >= s.r_min && r <= s.r_max && cnt[r] > 0) {
+        acc += (long long)r * pad8(cnt[r]);
+        tiles += (int)((pad8(cnt[r]) + 127) / 128);
+      }
+    }
+    base[kMaxR + 1] = acc;
+    tiles_pre[kMaxR + 1] = tiles;
+  }
+  __syncthreads();
+  const bool ok = base[kMaxR + 1] <= s.cap && qb[kMaxR + 1] <= qcap;
+  if (blockIdx.x == 0 && z == 0) {
+    for (int r = tid; r <= kMaxR + 1; r += blockDim.x) {
+      if (r <= kMaxR) cnt_out[(int64_t)b * (kMaxR + 1) + r] = cnt[r];
+      base_out[(int64_t)b * (kMaxR + 2) + r] = (r == kMaxR + 1 && !ok) ? -1 : base[r];
+    }
+    if (!ok && tid == 0) raise_status(dev_status, VARRATE_ERR_CORRUPT);
+  }
+  if (!ok) return;
+  const int64_t stream_q = (bl * s.G + g) * 2 + kv;
+  const int64_t stream_o = ((int64_t)b * s.G + g) * 2 + kv;
+  const uint8_t* src = qdata + stream_q * qcap;
+  __nv_bfloat16* dst = coef + stream_o * s.cap;
+  const int total = tiles_pre[kMaxR + 1];
+  const int T0 = (int)((long long)total * z / kDeqSplit), T1 = (int)((long long)total * (z + 1) / kDeqSplit);
+  const int lr = lane >> 4, gp = lane & 15;
+  for (int T = T0 + warp; T < T1; T += blockDim.x / 32) {
+    int lo_r = 0, hi_r = kMaxR + 1;   // tiles_pre[lo_r] <= T < tiles_pre[hi_r]
+    while (hi_r - lo_r > 1) {
+      const int mid = (lo_r + hi_r) >> 1;
+      if (tiles_pre[mid] <= T) lo_r = mid; else hi_r = mid;
+    }
+    const int r = lo_r;
+    const long long i = T - tiles_pre[r];
+    const int tl = (int)min(128ll, pad8(cnt[r]) - 128 * i);
+    const int ng = tl >> 3;
+    const int qrow = qrow_bytes(tl, BITS);
+    const uint8_t* qtile = src + qb[r] + i * (long long)r * qrow_bytes(128, BITS);
+    __nv_bfloat16* otile = dst + base[r] + 128 * i * r;
+    const bool full = ng == 16;   // warp-uniform: position (gp + j) mod 16 by a mask
+    const bool on = gp < ng;
+    // rows in batches of 2 x kDeqRows: every load of a batch is issued before the first use, so a
+    // warp keeps kDeqRows code words and group parameters per lane in flight
+    for (int j0 = 0; j0 < r; j0 += 2 * kDeqRows) {
+      typename CodeWord<BITS>::T w[kDeqRows];
+      uint32_t par[kDeqRows];
+#pragma unroll
+      for (int u = 0; u < kDeqRows; ++u) {
+        const int j = j0 + 2 * u + lr;
+        if (on && j < r) {
+          const uint8_t* row = qtile + (long long)j * qrow;
+          w[u] = *reinterpret_cast<const typename CodeWord<BITS>::T*>(row + (BITS == 4 ? 4 : 8) * gp);
+          par[u] = *reinterpret_cast<const uint32_t*>(row + tl * BITS / 8 + 4 * (gp >> 2));
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < kDeqRows; ++u) {
+        const int j = j0 + 2 * u + lr;
+        if (on && j < r) {
+          uint32_t c[8];
+          CodeWord<BITS>::unpack(w[u], c);
+          const __half2 ph = *reinterpret_cast<const __half2*>(&par[u]);
+          const float lo = __low2float(ph), st = __high2float(ph);
+          uint32_t o[4];
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {   // lo + code * step in one fused rounding, then bf16
+            const __nv_bfloat162 v = __floats2bfloat162_rn(fmaf((float)c[2 * e], st, lo),
+                                                           fmaf((float)c[2 * e + 1], st, lo));
+            o[e] = *reinterpret_cast<const uint32_t*>(&v);
+          }
+          const int pos = full ? ((gp + j) & 15) : (gp + j) % ng;
+          *reinterpret_cast<uint4*>(otile + (long long)j * tl + 8 * pos) = make_uint4(o[0], o[1], o[2], o[3]);
+        }
+      }
+    }
   }
 }
 
 }  // namespace
 
+size_t decode_q_expand_ws_bytes(const Shape& s, int num_sms) {
+  Shape s1 = s;
+  s1.L = 1;
+  const size_t dws = decode_ws_bytes(s1, num_sms);
+  const size_t coef = ((size_t)s.B * s.G * 2 * (size_t)s.cap * 2 + 255) & ~size_t(255);
+  const size_t cnt = ((size_t)s.B * (kMaxR + 1) * 4 + 255) & ~size_t(255);
+  const size_t base = ((size_t)s.B * (kMaxR + 2) * 8 + 255) & ~size_t(255);
+  return dws + coef + cnt + base;
+}
+
+bool decode_q_expand_supported(const Shape& s, int n_tail, int num_sms) {
+  Shape s1 = s;
+  s1.L = 1;
+  return s.dtype == VARRATE_BF16 && decode_mma_supported(s1, n_tail, num_sms) && s.B <= 65535;
+}
+
+int launch_decode_q_expand(const Shape& s, const varrate_qpacked& cache, const void* basis_k,
+                           const void* basis_v, const void* q, int layer, const void* tail_k,
+                           const void* tail_v, int n_tail, void* out, int32_t* dev_status, void* ws,
+                           int num_sms, cudaStream_t st) {
+  Shape s1 = s;
+  s1.L = 1;
+  char* w = static_cast<char*>(ws);
+  const size_t dws = decode_ws_bytes(s1, num_sms);
+  __nv_bfloat16* coef = reinterpret_cast<__nv_bfloat16*>(w + dws);
+  const size_t coef_b = ((size_t)s.B * s.G * 2 * (size_t)s.cap * 2 + 255) & ~size_t(255);
+  int32_t* cnt = reinterpret_cast<int32_t*>(w + dws + coef_b);
+  const size_t cnt_b = ((size_t)s.B * (kMaxR + 1) * 4 + 255) & ~size_t(255);
+  int64_t* base = reinterpret_cast<int64_t*>(w + dws + coef_b + cnt_b);
+  const dim3 grid(2 * s.G, s.B, kDeqSplit);
+  if (cache.bits == 4)
+    dequant_layer_kernel<4><<<grid, 256, 0, st>>>(cache.data, cache.qbase, cache.bucket_count, coef, cnt,
+                                                  base, dev_status, s, layer, cache.qcap_bytes);
+  else
+    dequant_layer_kernel<8><<<grid, 256, 0, st>>>(cache.data, cache.qbase, cache.bucket_count, coef, cnt,
+                                                  base, dev_status, s, layer, cache.qcap_bytes);
+  varrate_packed view = {};
+  view.coef = coef;
+  view.bucket_count = cnt;
+  view.bucket_base = base;
+  view.cap_elems = s.cap;
+  const size_t bstride = (size_t)layer * s.G * kHeadDim * kHeadDim;
+  const int rc = launch_decode(s1, view, static_cast<const __nv_bfloat16*>(basis_k) + bstride,
+                               static_cast<const __nv_bfloat16*>(basis_v) + bstride, q, 0, tail_k, tail_v,
+                               n_tail, out, dev_status, ws, num_sms, st);
+  return rc < 0 ? rc : rc + 1;
+}
+
 int launch_quantize(const Shape& s, const varrate_packed& in, const varrate_qpacked& out,
                     int32_t* dev_status, cudaStream_t st) {
   const int64_t pairs = (int64_t)s.B * s.L;
   qtables_kernel<<<(unsigned)((pairs + 127) / 128), 128, 0, st>>>(in.bucket_count, out.qbase, s, out.bits);
-  const dim3 grid(2 * s.G, (unsigned)pairs);
+  const dim3 grid(2 * s.G, (unsigned)pairs, kQuantSplit);
   if (out.bits == 4)
     quantize_kernel<4><<<grid, 256, 0, st>>>((const __nv_bfloat16*)in.coef, in.bucket_count,
                                              in.bucket_base, out.qbase, out.data, dev_status, s,

@@ -37,7 +37,7 @@ OK, FLOOR_BINDS = 0, 1
 ERR_ARG, ERR_WORKSPACE, ERR_CUDA, ERR_TIMEOUT, ERR_UNSUPPORTED, ERR_CORRUPT = -1, -2, -3, -4, -5, -6
 F32, BF16 = 0, 1
 SALIENCE, UNIFORM = 0, 1
-CALL_SALIENCE, CALL_PACK, CALL_ENCODE, CALL_DECODE, CALL_DECODE_WINDOW = 0, 1, 2, 3, 4
+CALL_SALIENCE, CALL_PACK, CALL_ENCODE, CALL_DECODE, CALL_DECODE_WINDOW, CALL_DECODE_Q = 0, 1, 2, 3, 4, 5
 
 _c_void_p = ctypes.c_void_p
 

@@ -129,14 +129,19 @@ def test_quantize_bit_exact(name, bits):
                 np.testing.assert_array_equal(st[mask].view(np.uint16), want[2][mask].view(np.uint16))
 
 
-@pytest.mark.parametrize("bits,n_tail", [(4, 0), (8, 0), (4, 37)])
+# workspace CALL_DECODE: the general kernels on x^ (fp32); CALL_DECODE_Q: the layer expanded to
+# bf16, then the fused tensor-core decode (beyond 256 tail tokens the general kernels again)
+@pytest.mark.parametrize("bits,n_tail,which", [(4, 0, "DECODE"), (8, 0, "DECODE"), (4, 37, "DECODE"),
+                                               (4, 0, "DECODE_Q"), (8, 0, "DECODE_Q"),
+                                               (4, 37, "DECODE_Q"), (8, 256, "DECODE_Q"),
+                                               (4, 300, "DECODE_Q")])
 @pytest.mark.parametrize("name", list(CASES))
-def test_decode_on_quantized_cache(name, bits, n_tail):
+def test_decode_on_quantized_cache(name, bits, n_tail, which):
     wl, cfg, bk, bv, refs, packed, coefs, pairs = _setup(name)
     qp = V.QPackedCache.allocate(cfg, packed, bits)
     status = torch.zeros(1, dtype=torch.int32, device="cuda")
     V.check(V.varrate_quantize(cfg, packed, qp, status), "varrate_quantize")
-    ws = V.workspace(cfg, V.CALL_DECODE)
+    ws = V.workspace(cfg, getattr(V, "CALL_" + which))
     gen = torch.Generator().manual_seed(11)
     worst = (0.0, 0.0)
     for l in range(wl.n_layers):
@@ -165,7 +170,7 @@ def test_decode_on_quantized_cache(name, bits, n_tail):
                                  None if tv is None else f64(tv[b]))
             assert decode_close(got[b], want, cfg), (l, b, decode_errors(got[b], want))
             worst = tuple(max(a, e) for a, e in zip(worst, decode_errors(got[b], want)))
-    print(f"{name} {bits}-bit: decode worst relative / absolute error {worst[0]:.3e} / {worst[1]:.3e}")
+    print(f"{name} {bits}-bit ({which}): decode worst relative / absolute error {worst[0]:.3e} / {worst[1]:.3e}")
 
 
 def test_quantized_round_trip_bound_at_full_size():
