@@ -111,3 +111,39 @@ def test_llama32_pack_full_size(llama32):
 def test_long_context_encode_and_decode(long_ctx):
     _check_encode(long_ctx)
     _check_decode(long_ctx, n_steps=1)
+
+
+def test_long_context_window_decode(long_ctx):
+    """The window call of the reuse workload (N = 131072, 32 window queries x GQA 4 = 128 query rows
+    per KV head, exact tail = the window's own 32 tokens), in the launch configuration bench.py
+    times. Sampled queries against the oracle with each query's causal cut of the tail, and the
+    score-blind control failing the same bar."""
+    import torch
+    wl, cfg, r = long_ctx["wl"], long_ctx["cfg"], long_ctx["gpu"]
+    _, _, _, bk, bv = long_ctx["inputs"]
+    ref = long_ctx["refs"][(0, 0)]
+    n_q = 32
+    q = synth.stack_decode_queries(wl, 0, n_q).permute(1, 0, 2, 3).contiguous()   # [B][n_q][H][d]
+    g = torch.Generator().manual_seed(5)
+    shape = (wl.batch, wl.n_kv_heads, n_q, wl.head_dim)
+    tk = torch.randn(shape, generator=g).to(torch.bfloat16)
+    tv = torch.randn(shape, generator=g).to(torch.bfloat16)
+    out = torch.empty_like(q, device="cuda")
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    ws = V.workspace(cfg, V.CALL_DECODE_WINDOW, "cuda")
+    V.check(V.varrate_decode_window(cfg, r["packed"], bk.cuda(), bv.cuda(), q.cuda(), n_q, 0,
+                                    tk.cuda(), tv.cuda(), n_q, out, status, ws),
+            "varrate_decode_window")
+    torch.cuda.synchronize()
+    assert int(status.item()) == V.OK
+    got = f64(out)
+    blind = uniform_weight_output(ref, f64(bv[0]), wl.group)
+    worst = (0.0, 0.0)
+    for i in (0, 13, n_q - 1):
+        m = i + 1                                 # tail tokens visible to query i
+        want = O.decode_coef(f64(q[0, i]), ref["coef_k"], ref["coef_v"], ref["ranks"], f64(bk[0]),
+                             f64(bv[0]), f64(tk[0, :, :m]), f64(tv[0, :, :m]))
+        assert decode_close(got[0, i], want, cfg), (i, decode_errors(got[0, i], want))
+        assert not decode_close(blind, want, cfg), (i, decode_errors(blind, want))
+        worst = tuple(max(a, e) for a, e in zip(worst, decode_errors(got[0, i], want)))
+    print(f"N={wl.n_ctx} window of {n_q}: worst relative / absolute error {worst[0]:.3e} / {worst[1]:.3e}")

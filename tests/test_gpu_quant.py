@@ -223,3 +223,43 @@ def test_quantized_round_trip_bound_at_full_size():
                         xmax = np.abs(x.reshape(-1, 8)).max()
                         bound = 0.5 * st32[grp] + 2.0 ** -10 * max(xmax, 1e-30)
                         assert np.all(np.abs(xh - x) <= bound), (bits, r, t0, j)
+
+
+def test_quantized_decode_full_size():
+    """llama32 layer call (8 sequences x 8 KV heads x N = 32768, GPU encode), 4-bit, through the
+    fused path (layer expanded to bf16, then the tensor-core decode) in the launch configuration
+    bench.py times: one sampled sequence against the oracle's decode on its own quantization of the
+    same stored coefficients, and a score-blind output failing the same bar."""
+    from gpu_helpers import uniform_weight_output, unpack
+    wl = synth.workload("llama32", n_layers=1)
+    k, v, qw, bk, bv = synth.stack_inputs(wl, device="cuda")
+    cfg = cfg_for(wl)
+    packed = V.PackedCache.allocate(cfg, "cuda")
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    V.check(V.varrate_encode(cfg, qw, k, v, bk, bv, None, packed, None, status,
+                             V.workspace(cfg, V.CALL_ENCODE)))
+    del k, v, qw
+    qp = V.QPackedCache.allocate(cfg, packed, 4)
+    V.check(V.varrate_quantize(cfg, packed, qp, status))
+    q = synth.stack_decode_queries(wl, 0, 1)[0]
+    out = torch.empty_like(q, device="cuda")
+    V.check(V.varrate_decode_attn_q(cfg, qp, bk, bv, q.cuda(), 0, None, None, 0, out, status,
+                                    V.workspace(cfg, V.CALL_DECODE_Q)), "varrate_decode_attn_q")
+    torch.cuda.synchronize()
+    assert int(status.item()) == V.OK
+    b = 3
+    ranks = packed.ranks[b, 0].cpu().numpy().astype(np.int64)
+    count = packed.bucket_count[b, 0].cpu().numpy()
+    base = packed.bucket_base[b, 0].cpu().numpy()
+    pos = packed.pos[b, 0].cpu().numpy()
+    deq = np.zeros((2, wl.n_kv_heads, wl.n_ctx, wl.head_dim))
+    for g in range(wl.n_kv_heads):
+        for kv in range(2):
+            stored = unpack(packed, b, 0, g, kv, ranks, count, base, pos).astype(np.float32)
+            deq[kv, g] = O.quantize_coefficients(stored, ranks, count, pos, 4)[3]
+    want = O.decode_coef(f64(q[b]), deq[0], deq[1], ranks, f64(bk[0]), f64(bv[0]))
+    got = f64(out)[b]
+    assert decode_close(got, want, cfg), decode_errors(got, want)
+    blind = uniform_weight_output(dict(coef_v=deq[1], ranks=ranks), f64(bv[0]), wl.group)
+    assert not decode_close(blind, want, cfg), decode_errors(blind, want)
+    print(f"llama32 4-bit fused: worst relative / absolute error {decode_errors(got, want)}")
