@@ -165,7 +165,7 @@ __device__ __forceinline__ void rot_compute(SegSmem& sm, const RotRegs& rr, int 
 }
 
 // Score-MMA B fragments of q~ (split hi + lo) for every 16-row chunk, one uint4 per lane.
-__device__ void build_qfrag(SegSmem& sm, int tid) {
+__device__ __noinline__ void build_qfrag(SegSmem& sm, int tid) {
   for (int i = tid; i < (kHeadDim / 16) * 32; i += NW * 32) {
     const int jc = i / 32, lane = i % 32, g8 = lane >> 2, c = lane & 3;
     const int j = jc * 16 + 2 * c;
@@ -220,7 +220,9 @@ static_assert(NW >= kHeadsPad, "one warp per head in the combine");
 // bf16 products of key and query); the tail's values join the rotation as further k-steps:
 //   out^T[col][head] = sum_j U_V[j][col] o~[head][j] + sum_t v_t[col] w[head][t]
 // with o~ and the tail weights w split hi + lo in bf16. Returns false if a staging copy timed out.
-__device__ bool combine_segment(CombSmem& cs, uint64_t* bar, uint32_t parity, const float* __restrict__ part,
+// Kept out of line (as is build_qfrag): the item loop's code stays compact (measured -0.2 us per
+// llama32 layer call).
+__device__ __noinline__ bool combine_segment(CombSmem& cs, uint64_t* bar, uint32_t parity, const float* __restrict__ part,
                                 int c0, int c1, long long seg, const __nv_bfloat16* __restrict__ q,
                                 const __nv_bfloat16* __restrict__ Uv, const __nv_bfloat16* __restrict__ tail_k,
                                 const __nv_bfloat16* __restrict__ tail_v, int n_tail,
