@@ -23,7 +23,7 @@
 //        values  O~^T[j][row] += V[j][slot] P^T[slot][row]      (P in bf16)
 //     The teams' states merge in shared memory into one partial (m, l, o~[128]) per row, per
 //     (segment, CTA).
-//  3. window_combine_kernel: per (sequence, KV head) and 16 rows, merges the partials of the CTAs
+//  3. window_combine_kernel: per (sequence, KV head) and 8 rows, merges the partials of the CTAs
 //     that shared the segment, adds the causal exact tail (scores and values in fp32 on CUDA
 //     cores, 64 tokens at a time, online), rotates o~ back with U_V^T and normalises.
 //
@@ -80,67 +80,83 @@ constexpr size_t win_smem_bytes() {
 
 // ------------------------------------------------------------------ 1. rotated query fragments
 
-// grid (B G, RG), 256 threads. CTA (seg, rg) computes q~ for the 16 rows of row group rg (n-tiles
-// rg and rg + RG; rows past R are zero) and writes them as fragments
-//   qf[seg][rg][jc][u][lane] = {hi(b0), hi(b1), lo(b0), lo(b1)}   (uint4)
+// grid (B G, RG, 4), 256 threads. CTA (seg, rg, z) computes q~[rho][j] for the 16 rows of row group
+// rg (n-tiles rg and rg + RG; rows past R are zero) and the 32 coefficients j in [32 z, 32 z + 32),
+// and writes them as fragments
+//   qf[seg][rg][jc][u][lane] = {hi(b0), hi(b1), lo(b0), lo(b1)}   (uint4, jc = 2 z, 2 z + 1)
 // with b0 = (q~[rho][16 jc + 2c], q~[rho][16 jc + 2c + 1]), b1 the same 8 columns later,
 // rho = 8 n-tile(u) + lane / 4, c = lane % 4: the B operand of m16n8k16 for k = 16 jc .. 16 jc + 15.
+constexpr int kQfJ = 32;   // coefficients per CTA
 __global__ void __launch_bounds__(256)
 window_qfrag_kernel(const __nv_bfloat16* __restrict__ basis_k, const __nv_bfloat16* __restrict__ q,
                     uint4* __restrict__ qf, Shape s, int layer, int n_q, int rg_count, int ntt) {
-  extern __shared__ __align__(16) unsigned char smem_q[];
-  float* ut = reinterpret_cast<float*>(smem_q);               // [128][129]: U_K transposed
-  float* qs = ut + kHeadDim * (kHeadDim + 1);                 // [16][128] query rows
-  float* qt = qs + 16 * kHeadDim;                             // [16][132] rotated rows
+  __shared__ float ut[kHeadDim][kQfJ + 1];   // U_K rows 32 z .. 32 z + 31, transposed
+  __shared__ float qs[16][kHeadDim];         // query rows
+  __shared__ float qt[16][kQfJ + 1];         // rotated rows
   const int tid = threadIdx.x;
   const long long seg = blockIdx.x;
-  const int rg = blockIdx.y;
+  const int rg = blockIdx.y, z = blockIdx.z;
   const int b = (int)(seg / s.G), g = (int)(seg % s.G);
   const int R = n_q * s.grp;
   pdl_trigger();
   pdl_wait();
-  const __nv_bfloat16* U = basis_k + ((long long)layer * s.G + g) * kHeadDim * kHeadDim;
-  for (int e = tid; e < kHeadDim * kHeadDim / 2; e += blockDim.x) {
-    const int j = e / (kHeadDim / 2), i = 2 * (e % (kHeadDim / 2));
-    const __nv_bfloat162 u = reinterpret_cast<const __nv_bfloat162*>(U)[e];
-    ut[i * (kHeadDim + 1) + j] = __low2float(u);
-    ut[(i + 1) * (kHeadDim + 1) + j] = __high2float(u);
+  const __nv_bfloat16* U = basis_k + ((long long)layer * s.G + g) * kHeadDim * kHeadDim + (long long)z * kQfJ * kHeadDim;
+  // 32 rows x 128 bf16 = 512 uint4: two per thread, both loads in flight
+  {
+    const uint4* u4 = reinterpret_cast<const uint4*>(U);
+    const uint4 v0 = __ldg(u4 + tid), v1 = __ldg(u4 + tid + 256);
+    const uint4 vv[2] = {v0, v1};
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int e = tid + 256 * h, j = e >> 4, i0 = (e & 15) * 8;
+      const uint32_t w[4] = {vv[h].x, vv[h].y, vv[h].z, vv[h].w};
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        ut[i0 + 2 * k][j] = __uint_as_float(w[k] << 16);
+        ut[i0 + 2 * k + 1][j] = __uint_as_float(w[k] & 0xffff0000u);
+      }
+    }
   }
-  // local row l: n-tile rg (l < 8) or rg + RG, row 8 * nt + l % 8
-  for (int e = tid; e < 16 * kHeadDim; e += blockDim.x) {
-    const int l = e / kHeadDim, i = e % kHeadDim;
+  // local row l: n-tile rg (l < 8) or rg + RG, row 8 * nt + l % 8; 16 rows x 16 uint4
+  {
+    const int l = tid >> 4, c4 = tid & 15;
     const int nt = l < 8 ? rg : rg + rg_count;
     const int rho = 8 * nt + (l & 7);
-    float v = 0.f;
+    uint4 v = make_uint4(0u, 0u, 0u, 0u);
     if (nt < ntt && rho < R) {
       const int iq = rho / s.grp, h = rho % s.grp;
-      v = __bfloat162float(q[(((long long)b * n_q + iq) * s.H + (long long)g * s.grp + h) * kHeadDim + i]);
+      v = __ldg(reinterpret_cast<const uint4*>(q + (((long long)b * n_q + iq) * s.H + (long long)g * s.grp + h) * kHeadDim) + c4);
     }
-    qs[e] = v;
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      qs[l][c4 * 8 + 2 * k] = __uint_as_float(w[k] << 16);
+      qs[l][c4 * 8 + 2 * k + 1] = __uint_as_float(w[k] & 0xffff0000u);
+    }
   }
   __syncthreads();
-  {
-    const int j = tid & (kHeadDim - 1), l0 = (tid >> 7) * 8;
-    float acc[8] = {};
+  {   // thread: coefficient j = tid % 32, rows l0 .. l0 + 1 (l0 = 2 (tid / 32))
+    const int j = tid & (kQfJ - 1), l0 = (tid >> 5) * 2;
+    float a0 = 0.f, a1 = 0.f;
+#pragma unroll 8
     for (int i = 0; i < kHeadDim; ++i) {
-      const float u = ut[i * (kHeadDim + 1) + j];
-#pragma unroll
-      for (int r = 0; r < 8; ++r) acc[r] = fmaf(u, qs[(l0 + r) * kHeadDim + i], acc[r]);
+      const float u = ut[i][j];
+      a0 = fmaf(u, qs[l0][i], a0);
+      a1 = fmaf(u, qs[l0 + 1][i], a1);
     }
     const float scale = kLog2e * rsqrtf((float)kHeadDim);
-#pragma unroll
-    for (int r = 0; r < 8; ++r) qt[(l0 + r) * (kHeadDim + 4) + j] = acc[r] * scale;
+    qt[l0][j] = a0 * scale;
+    qt[l0 + 1][j] = a1 * scale;
   }
   __syncthreads();
-  uint4* dst = qf + (seg * rg_count + rg) * kQfWords;
-  for (int e = tid; e < kQfWords; e += blockDim.x) {
-    const int jc = e / 64, u = (e / 32) & 1, lane = e & 31;
-    const int l = u * 8 + (lane >> 2), j = jc * 16 + 2 * (lane & 3);
-    const float* row = qt + l * (kHeadDim + 4);
+  uint4* dst = qf + (seg * rg_count + rg) * kQfWords + (long long)z * 2 * 2 * 32;
+  if (tid < 2 * 2 * 32) {
+    const int jl = tid / 64, u = (tid / 32) & 1, lane = tid & 31;   // jc = 2 z + jl
+    const int l = u * 8 + (lane >> 2), j = jl * 16 + 2 * (lane & 3);
     uint32_t h0, l0, h1, l1;
-    split_bf16(row[j], row[j + 1], h0, l0);
-    split_bf16(row[j + 8], row[j + 9], h1, l1);
-    dst[e] = make_uint4(h0, h1, l0, l1);
+    split_bf16(qt[l][j], qt[l][j + 1], h0, l0);
+    split_bf16(qt[l][j + 8], qt[l][j + 9], h1, l1);
+    dst[tid] = make_uint4(h0, h1, l0, l1);
   }
 }
 
@@ -600,21 +616,22 @@ decode_window_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __re
 
 // ------------------------------------------------------------------ 3. combine
 
-constexpr int kTT = 64;              // tail tokens per step
+constexpr int kTT = 64;                   // tail tokens per step
 constexpr int kKsStride = kHeadDim + 2;   // staged tail keys (odd word stride: no bank conflicts)
+constexpr int kCombRows = 8;              // query rows per combine CTA: one warp each
 
 struct CombineSmem {
   __nv_bfloat16 us[kHeadDim * kHeadDim];   // U_V[j][col]
   __nv_bfloat16 ks[kTT * kKsStride];        // tail keys of the step
   __nv_bfloat16 vs[kTT * kHeadDim];         // tail values of the step
-  float qs[16][kHeadDim];                   // raw query rows (fp32)
-  float os[16][kHeadDim + 4];               // merged o~ per row
-  float ws[16][kTT];                        // tail weights of the step
+  float qs[kCombRows][kHeadDim];            // raw query rows (fp32)
+  float os[kCombRows][kHeadDim + 4];        // merged o~ per row
+  float ws[kCombRows][kTT];                 // tail weights of the step
 };
 
-// grid (B G, ceil(R / 16)), 256 threads: thread (lr = tid / 16, cl = tid % 16) owns row
-// rho = 16 blockIdx.y + lr and columns cl + 16 k (k < 8). part slots as written above; out is
-// [B][n_q][H][d].
+// grid (B G, ceil(R / 8)), 256 threads: warp w owns row rho = 8 blockIdx.y + w, lane l its columns
+// l + 32 k (k < 4) and, per step of 64 tail tokens, tokens l and l + 32. part slots as written
+// above; out is [B][n_q][H][d].
 __global__ void __launch_bounds__(256)
 window_combine_kernel(const float* __restrict__ part, const int64_t* __restrict__ bucket_base,
                       const __nv_bfloat16* __restrict__ basis_v, const __nv_bfloat16* __restrict__ q,
@@ -625,54 +642,60 @@ window_combine_kernel(const float* __restrict__ part, const int64_t* __restrict_
   CombineSmem& cs = *reinterpret_cast<CombineSmem*>(smem_c);
   __shared__ long long segW[64];
   __shared__ long long segP[65];
-  const int tid = threadIdx.x, lr = tid >> 4, cl = tid & 15;
+  const int tid = threadIdx.x, lr = tid >> 5, lane = tid & 31;
   const long long seg = blockIdx.x;
   const int b = (int)(seg / s.G), g = (int)(seg % s.G);
   const int R = n_q * s.grp, rows = 8 * ntt;
-  const int rho = 16 * blockIdx.y + lr;
+  const int rho = kCombRows * blockIdx.y + lr;
   const bool valid = rho < R;
   const int iq = valid ? rho / s.grp : 0, h = valid ? rho % s.grp : 0;
   pdl_trigger();
   pdl_wait();
-  // U_V of the head and the query rows: plain loads, consumed at the end / by the tail scores
+  // U_V of the head (eight 16-byte loads per thread, all in flight) and the query rows
   {
     const uint4* src = reinterpret_cast<const uint4*>(basis_v + ((long long)layer * s.G + g) * kHeadDim * kHeadDim);
     uint4* dst = reinterpret_cast<uint4*>(cs.us);
-    for (int e = tid; e < kHeadDim * kHeadDim / 8; e += blockDim.x) dst[e] = src[e];
-    for (int e = tid; e < 16 * kHeadDim; e += blockDim.x) {
-      const int l = e / kHeadDim, i = e % kHeadDim, rr = 16 * blockIdx.y + l;
-      float v = 0.f;
-      if (rr < R)
-        v = __bfloat162float(q[(((long long)b * n_q + rr / s.grp) * s.H + (long long)g * s.grp + rr % s.grp) * kHeadDim + i]);
-      cs.qs[l][i] = v;
-    }
+    uint4 v[kHeadDim * kHeadDim / 8 / 256];
+#pragma unroll
+    for (int k = 0; k < kHeadDim * kHeadDim / 8 / 256; ++k) v[k] = __ldg(src + tid + 256 * k);
+#pragma unroll
+    for (int k = 0; k < kHeadDim * kHeadDim / 8 / 256; ++k) dst[tid + 256 * k] = v[k];
+    const __nv_bfloat16* qr = q + (((long long)b * n_q + iq) * s.H + (long long)g * s.grp + h) * kHeadDim;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) cs.qs[lr][lane + 32 * k] = valid ? __bfloat162float(qr[lane + 32 * k]) : 0.f;
   }
   seg_lengths(bucket_base, s, layer, segW, segP, tid);
-  // merge the partials of the CTAs that shared the segment
-  float M = -INFINITY, L = 0.f, o[8], ov[8];
+  // merge the partials of the CTAs that shared the segment: the common maximum first, then the
+  // weighted sums (independent loads, four partials at a time)
+  float M = -INFINITY, L = 0.f, o[4], ov[4];
 #pragma unroll
-  for (int k = 0; k < 8; ++k) { o[k] = 0.f; ov[k] = 0.f; }
+  for (int k = 0; k < 4; ++k) { o[k] = 0.f; ov[k] = 0.f; }
   const long long W = segW[b];
   if (W > 0 && valid) {
     const long long T = segP[64];
     const long long P = segP[b] + g * (W + kSegCost + kSegEnd) + kSegCost;
     int c0, c1;
     seg_cta_range([&](int i) { return cut_at(T, i, C); }, T, C, P, W, c0, c1);
-    for (int p = c0; p <= c1; ++p) {
-      const float* pp = part + ((p + seg) * (long long)rows + rho) * kPartStride;
-      const float mp = __ldcg(pp + kHeadDim), lp = __ldcg(pp + kHeadDim + 1);
-      if (mp == -INFINITY) continue;
-      const float nm = fmaxf(M, mp);
-      const float f = M == -INFINITY ? 0.f : exp2f(M - nm), fp = exp2f(mp - nm);
+    const float* pr = part + ((c0 + seg) * (long long)rows + rho) * kPartStride;
+    const long long pstride = (long long)rows * kPartStride;
+    const int np = c1 - c0 + 1;
+#pragma unroll 4
+    for (int p = 0; p < np; ++p) M = fmaxf(M, __ldcg(pr + p * pstride + kHeadDim));
+    if (M != -INFINITY) {
+#pragma unroll 4
+      for (int p = 0; p < np; ++p) {
+        const float* pp = pr + p * pstride;
+        const float mp = __ldcg(pp + kHeadDim);
+        const float w = mp == -INFINITY ? 0.f : exp2f(mp - M);
+        L = fmaf(w, __ldcg(pp + kHeadDim + 1), L);
 #pragma unroll
-      for (int k = 0; k < 8; ++k) o[k] = fmaf(fp, __ldcg(pp + cl + 16 * k), o[k] * f);
-      L = fmaf(fp, lp, L * f);
-      M = nm;
+        for (int k = 0; k < 4; ++k) o[k] = fmaf(w, __ldcg(pp + lane + 32 * k), o[k]);
+      }
     }
   }
   // exact tail, causal: row rho (query iq) sees tail tokens t < n_tail - n_q + iq + 1
   const int vis = n_tail - n_q + iq + 1;
-  const int last_row = min(R, 16 * (int)blockIdx.y + 16) - 1;
+  const int last_row = min(R, kCombRows * (int)blockIdx.y + kCombRows) - 1;
   const int vis_max = n_tail - n_q + last_row / s.grp + 1;   // block-uniform
   const float scale = kLog2e * rsqrtf((float)kHeadDim);
   const __nv_bfloat16* tk = tail_k + ((long long)b * s.G + g) * n_tail * kHeadDim;
@@ -690,69 +713,71 @@ window_combine_kernel(const float* __restrict__ part, const int64_t* __restrict_
       reinterpret_cast<uint32_t*>(cs.vs + t * kHeadDim)[i2] = vx;
     }
     __syncthreads();
-    float sc[4] = {0.f, 0.f, 0.f, 0.f};
+    float sc[2] = {0.f, 0.f};
     for (int i = 0; i < kHeadDim; i += 2) {
       const float2 qv = *reinterpret_cast<const float2*>(&cs.qs[lr][i]);
 #pragma unroll
-      for (int k = 0; k < 4; ++k) {
-        const __nv_bfloat162 kk = *reinterpret_cast<const __nv_bfloat162*>(cs.ks + (cl + 16 * k) * kKsStride + i);
+      for (int k = 0; k < 2; ++k) {
+        const __nv_bfloat162 kk = *reinterpret_cast<const __nv_bfloat162*>(cs.ks + (lane + 32 * k) * kKsStride + i);
         sc[k] = fmaf(qv.x, __low2float(kk), fmaf(qv.y, __high2float(kk), sc[k]));
       }
     }
     float tm = -INFINITY;
 #pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      const int t = t0 + cl + 16 * k;
+    for (int k = 0; k < 2; ++k) {
+      const int t = t0 + lane + 32 * k;
       sc[k] = (valid && t < vis) ? sc[k] * scale : -INFINITY;
       tm = fmaxf(tm, sc[k]);
     }
 #pragma unroll
-    for (int x = 1; x < 16; x <<= 1) tm = fmaxf(tm, __shfl_xor_sync(0xffffffffu, tm, x));
+    for (int x = 1; x < 32; x <<= 1) tm = fmaxf(tm, __shfl_xor_sync(0xffffffffu, tm, x));
     const float nm = fmaxf(M, tm);
     float lt = 0.f;
     if (nm != -INFINITY) {
       const float f = M == -INFINITY ? 0.f : exp2f(M - nm);
 #pragma unroll
-      for (int k = 0; k < 8; ++k) { o[k] *= f; ov[k] *= f; }
+      for (int k = 0; k < 4; ++k) { o[k] *= f; ov[k] *= f; }
       L *= f;
       M = nm;
 #pragma unroll
-      for (int k = 0; k < 4; ++k) {
+      for (int k = 0; k < 2; ++k) {
         const float w = sc[k] == -INFINITY ? 0.f : exp2f(sc[k] - nm);
-        cs.ws[lr][cl + 16 * k] = w;
+        cs.ws[lr][lane + 32 * k] = w;
         lt += w;
       }
     } else {
 #pragma unroll
-      for (int k = 0; k < 4; ++k) cs.ws[lr][cl + 16 * k] = 0.f;
+      for (int k = 0; k < 2; ++k) cs.ws[lr][lane + 32 * k] = 0.f;
     }
 #pragma unroll
-    for (int x = 1; x < 16; x <<= 1) lt += __shfl_xor_sync(0xffffffffu, lt, x);
+    for (int x = 1; x < 32; x <<= 1) lt += __shfl_xor_sync(0xffffffffu, lt, x);
     L += lt;
-    __syncwarp();   // the 16 threads of a row are in one warp
+    __syncwarp();   // the row's weights were written by this warp
+#pragma unroll 4
     for (int t = 0; t < kTT; ++t) {
       const float w = cs.ws[lr][t];
 #pragma unroll
-      for (int k = 0; k < 8; ++k) ov[k] = fmaf(w, __bfloat162float(cs.vs[t * kHeadDim + cl + 16 * k]), ov[k]);
+      for (int k = 0; k < 4; ++k) ov[k] = fmaf(w, __bfloat162float(cs.vs[t * kHeadDim + lane + 32 * k]), ov[k]);
     }
   }
   // rotate the coded part back: out[col] = sum_j U_V[j][col] o~[j] + tail values, over l
 #pragma unroll
-  for (int k = 0; k < 8; ++k) cs.os[lr][cl + 16 * k] = o[k];
+  for (int k = 0; k < 4; ++k) cs.os[lr][lane + 32 * k] = o[k];
   __syncthreads();
-  float y[8];
+  float y[4];
 #pragma unroll
-  for (int k = 0; k < 8; ++k) y[k] = ov[k];
+  for (int k = 0; k < 4; ++k) y[k] = ov[k];
+#pragma unroll 4
   for (int j = 0; j < kHeadDim; ++j) {
     const float oj = cs.os[lr][j];
 #pragma unroll
-    for (int k = 0; k < 8; ++k) y[k] = fmaf(__bfloat162float(cs.us[j * kHeadDim + cl + 16 * k]), oj, y[k]);
+    for (int k = 0; k < 4; ++k) y[k] = fmaf(__bfloat162float(cs.us[j * kHeadDim + lane + 32 * k]), oj, y[k]);
   }
   if (valid) {
     __nv_bfloat16* dst = out + (((long long)b * n_q + iq) * s.H + (long long)g * s.grp + h) * kHeadDim;
     const float inv = 1.f / L;
 #pragma unroll
-    for (int k = 0; k < 8; ++k) dst[cl + 16 * k] = __float2bfloat16_rn(y[k] * inv);
+    for (int k = 0; k < 4; ++k) dst[lane + 32 * k] = __float2bfloat16_rn(y[k] * inv);
   }
 }
 
@@ -829,12 +854,10 @@ int launch_decode_window(const Shape& s, const varrate_packed& c, const void* ba
   pdl[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   pdl[0].val.programmaticStreamSerializationAllowed = 1;
 
-  const size_t qsm = (size_t)(kHeadDim * (kHeadDim + 1) + 16 * kHeadDim + 16 * (kHeadDim + 4)) * sizeof(float);
-  if (!helper_smem(0, (const void*)window_qfrag_kernel, qsm)) return -1;
   cudaLaunchConfig_t lq = {};
-  lq.gridDim = dim3((unsigned)segs, RG);
+  lq.gridDim = dim3((unsigned)segs, RG, kHeadDim / kQfJ);
   lq.blockDim = dim3(256);
-  lq.dynamicSmemBytes = qsm;
+  lq.dynamicSmemBytes = 0;
   lq.stream = st;
   lq.attrs = pdl;
   lq.numAttrs = 1;
@@ -854,7 +877,7 @@ int launch_decode_window(const Shape& s, const varrate_packed& c, const void* ba
   const size_t csm = sizeof(CombineSmem);
   if (!helper_smem(1, (const void*)window_combine_kernel, csm)) return -1;
   cudaLaunchConfig_t lc = {};
-  lc.gridDim = dim3((unsigned)segs, (unsigned)((R + 15) / 16));
+  lc.gridDim = dim3((unsigned)segs, (unsigned)((R + kCombRows - 1) / kCombRows));
   lc.blockDim = dim3(256);
   lc.dynamicSmemBytes = csm;
   lc.stream = st;
