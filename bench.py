@@ -69,10 +69,11 @@ def measured_traffic():
 
 
 def kernel_source_sha256():
-    """sha256 over the decode kernel's sources (decode_mma.cu, decode_common.cuh, common.cuh)."""
+    """sha256 over the decode kernel's sources (decode_mma.cu, decode_parts.cuh, decode_common.cuh,
+    common.cuh)."""
     import hashlib
     h = hashlib.sha256()
-    for name in ("decode_mma.cu", "decode_common.cuh", "common.cuh"):
+    for name in ("decode_mma.cu", "decode_parts.cuh", "decode_common.cuh", "common.cuh"):
         h.update(open(os.path.join(ROOT, "paper_2607_15498_gb300", "csrc", name), "rb").read())
     return h.hexdigest()
 
@@ -548,7 +549,7 @@ def sweep_quant(V, wl, dev, peak, stream, decode_steps, bits_list=(4, 8)):
     qdec = torch.stack([synth.stack_decode_queries(wl, l, decode_steps, device=dev)
                         for l in range(wl.n_layers)], dim=1)
     out = torch.empty((wl.batch, wl.n_q_heads, d), dtype=torch.bfloat16, device=dev)
-    ws = V.workspace(cfg, V.CALL_DECODE_Q, dev)   # room for the layer's bf16 expansion
+    ws = V.workspace(cfg, V.CALL_DECODE_Q, dev)
     res = {}
     for bits in bits_list:
         qp = V.QPackedCache.allocate(cfg, packed, bits, dev)
@@ -591,9 +592,9 @@ def sweep_quant(V, wl, dev, peak, stream, decode_steps, bits_list=(4, 8)):
             "decode_bytes_per_layer_call": int(step_bytes / wl.n_layers),
             "decode_gbs": round(gbs, 1), "decode_frac_of_hbm_peak": round(gbs / peak, 4),
             "decode_status": V.status_string(int(status.item())),
-            "decode_kernels": "per layer call: the layer expanded to bf16 in the workspace (one "
-                              "dequantize launch, writing 2 B per coefficient), then the fused "
-                              "tensor-core decode on it; graph-replayed"}
+            "decode_kernels": "per layer call: one fused kernel reading only the codes and their "
+                              "group parameters, dequantized in each warp's ring into fp16 tiles; "
+                              "graph-replayed"}
         del g, qp
     res["workload"] = workload_desc(wl)
     del packed, qdec

@@ -269,12 +269,15 @@ varrate_status varrate_quantize(const varrate_config* cfg, const varrate_packed*
 /* Decode attention of one layer on a quantized cache: the same mathematics and arguments as
  * varrate_decode_attn with each stored coefficient c replaced by its dequantized value x^
  * = fl32(lo + fl32(code * step)); 0 <= n_tail <= 4096; dtype VARRATE_BF16 only (queries, bases,
- * tail and output bf16). ws holds at least varrate_workspace_bytes(cfg, VARRATE_CALL_DECODE) bytes,
- * zero-filled before first use like the decode workspace (its header is the same).
- *  - With at least varrate_workspace_bytes(cfg, VARRATE_CALL_DECODE_Q) bytes and a shape the fused
- *    bf16 decode kernel takes (see varrate_decode_attn), the layer is first expanded into the
- *    workspace as a bf16 packed cache (x^ rounded to bf16) and then decoded by that kernel: two
- *    launches, the second with programmatic stream serialization as for varrate_decode_attn.
+ * tail and output bf16). ws holds at least varrate_workspace_bytes(cfg, VARRATE_CALL_DECODE) bytes
+ * (VARRATE_CALL_DECODE_Q asks for the same size), zero-filled before first use like the decode
+ * workspace (its header is the same).
+ *  - With n_tail <= 256, batch <= 64, batch * n_kv_heads <= 4096 and qcap_bytes a multiple of 16,
+ *    one fused kernel runs, with the shape limits and the programmatic stream serialization of the
+ *    fused kernel of varrate_decode_attn: it reads the codes and their group parameters (nothing
+ *    else of the cache) into shared memory, turns them into x^ rounded to fp16 (one fused
+ *    multiply-add from the exact code and the fp16 lo and step) and runs the tensor-core
+ *    attention on those fp16 values.
  *  - Otherwise the general kernels (query rotation, split over tokens, combine) decode on x^ in
  *    fp32 directly. */
 varrate_status varrate_decode_attn_q(const varrate_config* cfg, const varrate_qpacked* cache,

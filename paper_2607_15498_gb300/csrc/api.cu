@@ -88,7 +88,7 @@ size_t ws_bytes(const varrate_config* c, int32_t which) {
              align256((size_t)s.B * s.L * sizeof(int64_t));
     case VARRATE_CALL_DECODE: return vr::decode_ws_bytes(s, sms);
     case VARRATE_CALL_DECODE_WINDOW: return vr::decode_window_ws_bytes(s, sms);
-    case VARRATE_CALL_DECODE_Q: return std::max(vr::decode_ws_bytes(s, sms), vr::decode_q_expand_ws_bytes(s, sms));
+    case VARRATE_CALL_DECODE_Q: return vr::decode_ws_bytes(s, sms);
     default: return 0;
   }
 }
@@ -316,9 +316,11 @@ varrate_status varrate_decode_attn_q(const varrate_config* cfg, const varrate_qp
   if (ws_bytes_ < need || ws == nullptr) return VARRATE_ERR_WORKSPACE;
   const Shape s = make_shape(cfg, cap_elems(cfg));
   const int sms = num_sms();
-  if (vr::decode_q_expand_supported(s, n_tail, sms) && ws_bytes_ >= ws_bytes(cfg, VARRATE_CALL_DECODE_Q)) {
-    if (vr::launch_decode_q_expand(s, *cache, basis_k, basis_v, q, layer, tail_k, tail_v, n_tail, out,
-                                   dev_status, ws, sms, (cudaStream_t)stream) < 0)
+  if (vr::decode_q_supported(s, cache->bits, cache->qcap_bytes, n_tail, sms) && aligned16({cache->data})) {
+    char* w = static_cast<char*>(ws);
+    if (vr::launch_decode_q_fused(s, *cache, basis_k, basis_v, q, layer, tail_k, tail_v, n_tail, out, dev_status,
+                                  w, reinterpret_cast<float*>(w + vr::kDecodeCounterBytes), sms,
+                                  (cudaStream_t)stream) < 0)
       return VARRATE_ERR_CUDA;
     return launched();
   }

@@ -79,17 +79,18 @@ int launch_decode_window(const Shape& s, const varrate_packed& c, const void* ba
                          int n_tail, void* out, int32_t* dev_status, void* ws, int num_sms,
                          cudaStream_t st);
 
-// ---- quantized coefficients (quant.cu; decode with the general kernels in decode.cu)
+// ---- quantized coefficients (quant.cu)
 int launch_quantize(const Shape& s, const varrate_packed& in, const varrate_qpacked& out,
                     int32_t* dev_status, cudaStream_t st);
-// the fused path for quantized caches: the layer expanded to bf16 in the workspace, then the bf16
-// tensor-core decode (quant.cu); the workspace is the 1-layer decode workspace plus the expansion
-size_t decode_q_expand_ws_bytes(const Shape& s, int num_sms);
-bool decode_q_expand_supported(const Shape& s, int n_tail, int num_sms);
-int launch_decode_q_expand(const Shape& s, const varrate_qpacked& cache, const void* basis_k,
-                           const void* basis_v, const void* q, int layer, const void* tail_k,
-                           const void* tail_v, int n_tail, void* out, int32_t* dev_status, void* ws,
-                           int num_sms, cudaStream_t st);
+// Fused decode on a group-quantized cache (decode_q.cu): the bf16 kernel's work split with the
+// codes dequantized in each warp's ring. Workspace: that of the bf16 fused decode (header, then
+// the partials). Shapes it does not take run the general kernels on x^ (launch_decode_q,
+// decode.cu).
+bool decode_q_supported(const Shape& s, int bits, int64_t qcap, int n_tail, int num_sms);
+int launch_decode_q_fused(const Shape& s, const varrate_qpacked& cache, const void* basis_k,
+                          const void* basis_v, const void* q, int layer, const void* tail_k,
+                          const void* tail_v, int n_tail, void* out, int32_t* dev_status, void* header,
+                          float* part, int num_sms, cudaStream_t st);
 int launch_decode_q(const Shape& s, const varrate_qpacked& cache, const void* basis_k,
                     const void* basis_v, const void* q, int layer, const void* tail_k,
                     const void* tail_v, int n_tail, void* out, void* ws, int num_sms, cudaStream_t st);

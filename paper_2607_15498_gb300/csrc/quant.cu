@@ -47,7 +47,7 @@ __global__ void qtables_kernel(const int32_t* __restrict__ bucket_count, int64_t
 // writes its 8 codes (one 32-bit word at 4 bits, two at 8 bits); the group's first lane writes
 // (lo, step) and the row's padding bytes are zeroed.
 constexpr int kQuantSplit = 8;
-constexpr int kDeqRows = 8;   // rows per lane whose loads are in flight together (both directions)
+constexpr int kDeqRows = 8;   // rows per lane whose loads are in flight together
 
 template <int BITS>
 __global__ void __launch_bounds__(256)
@@ -162,184 +162,7 @@ quantize_kernel(const __nv_bfloat16* __restrict__ coef, const int32_t* __restric
   }
 }
 
-// Expansion of one layer of a quantized cache to the bf16 packed layout, for the fused decode:
-// grid (2 G, B, kDeqSplit), 256 threads. CTA (stream, b, z) writes the z-th share of the tiles of
-// stream (b, layer, g, kv); a warp takes one tile at a time, two rows per step: lane (lr, gp) turns
-// the 8 codes of slot group gp of row 2 jj + lr into lo + code * step (one fused multiply-add, within
-// an fp32 rounding of x^ = fl32(lo + fl32(code * step))), rounds them to bf16 and stores them as one 16-byte group at its packed position (group gp of row j at
-// position (gp + j) mod (tl / 8)). CTA (0, b, 0) also writes sequence b's bucket counts and element
-// bases for the layer (a table that does not fit the buffers is written as an empty stream and
-// raises VARRATE_ERR_CORRUPT).
-constexpr int kDeqSplit = 8;
-
-// The 8 codes of one 8-slot group: one 32-bit word (4-bit codes, the even slot in the low nibble)
-// or two (8-bit).
-template <int BITS> struct CodeWord;
-template <> struct CodeWord<4> {
-  using T = uint32_t;
-  static __device__ __forceinline__ void unpack(uint32_t w, uint32_t (&c)[8]) {
-#pragma unroll
-    for (int e = 0; e < 8; ++e) c[e] = (w >> (4 * e)) & 15u;
-  }
-};
-template <> struct CodeWord<8> {
-  using T = uint2;
-  static __device__ __forceinline__ void unpack(uint2 w, uint32_t (&c)[8]) {
-#pragma unroll
-    for (int e = 0; e < 4; ++e) { c[e] = (w.x >> (8 * e)) & 255u; c[4 + e] = (w.y >> (8 * e)) & 255u; }
-  }
-};
-
-template <int BITS>
-__global__ void __launch_bounds__(256)
-dequant_layer_kernel(const uint8_t* __restrict__ qdata, const int64_t* __restrict__ qbase,
-                     const int32_t* __restrict__ bucket_count, __nv_bfloat16* __restrict__ coef,
-                     int32_t* __restrict__ cnt_out, int64_t* __restrict__ base_out,
-                     int32_t* __restrict__ dev_status, Shape s, int layer, int64_t qcap) {
-  __shared__ int cnt[kMaxR + 1];
-  __shared__ long long base[kMaxR + 2];
-  __shared__ long long qb[kMaxR + 2];
-  __shared__ int tiles_pre[kMaxR + 2];   // tiles of the buckets before r
-  const int kv = blockIdx.x & 1, g = blockIdx.x >> 1, b = blockIdx.y, z = blockIdx.z;
-  const int64_t bl = (int64_t)b * s.L + layer;
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  for (int r = tid; r <= kMaxR + 1; r += blockDim.x) {
-    if (r <= kMaxR) cnt[r] = bucket_count[bl * (kMaxR + 1) + r];
-    qb[r] = qbase[bl * (kMaxR + 2) + r];
-  }
-  __syncthreads();
-  if (tid == 0) {
-    long long acc = 0;
-    int tiles = 0;
-    for (int r = 0; r <= kMaxR; ++r) {
-      base[r] = acc;
-      tiles_pre[r] = tiles;
-      if (r >= s.r_min && r <= s.r_max && cnt[r] > 0) {
-        acc += (long long)r * pad8(cnt[r]);
-        tiles += (int)((pad8(cnt[r]) + 127) / 128);
-      }
-    }
-    base[kMaxR + 1] = acc;
-    tiles_pre[kMaxR + 1] = tiles;
-  }
-  __syncthreads();
-  const bool ok = base[kMaxR + 1] <= s.cap && qb[kMaxR + 1] <= qcap;
-  if (blockIdx.x == 0 && z == 0) {
-    for (int r = tid; r <= kMaxR + 1; r += blockDim.x) {
-      if (r <= kMaxR) cnt_out[(int64_t)b * (kMaxR + 1) + r] = cnt[r];
-      base_out[(int64_t)b * (kMaxR + 2) + r] = (r == kMaxR + 1 && !ok) ? -1 : base[r];
-    }
-    if (!ok && tid == 0) raise_status(dev_status, VARRATE_ERR_CORRUPT);
-  }
-  if (!ok) return;
-  const int64_t stream_q = (bl * s.G + g) * 2 + kv;
-  const int64_t stream_o = ((int64_t)b * s.G + g) * 2 + kv;
-  const uint8_t* src = qdata + stream_q * qcap;
-  __nv_bfloat16* dst = coef + stream_o * s.cap;
-  const int total = tiles_pre[kMaxR + 1];
-  const int T0 = (int)((long long)total * z / kDeqSplit), T1 = (int)((long long)total * (z + 1) / kDeqSplit);
-  const int lr = lane >> 4, gp = lane & 15;
-  for (int T = T0 + warp; T < T1; T += blockDim.x / 32) {
-    int lo_r = 0, hi_r = kMaxR + 1;   // tiles_pre[lo_r] <= T < tiles_pre[hi_r]
-    while (hi_r - lo_r > 1) {
-      const int mid = (lo_r + hi_r) >> 1;
-      if (tiles_pre[mid] <= T) lo_r = mid; else hi_r = mid;
-    }
-    const int r = lo_r;
-    const long long i = T - tiles_pre[r];
-    const int tl = (int)min(128ll, pad8(cnt[r]) - 128 * i);
-    const int ng = tl >> 3;
-    const int qrow = qrow_bytes(tl, BITS);
-    const uint8_t* qtile = src + qb[r] + i * (long long)r * qrow_bytes(128, BITS);
-    __nv_bfloat16* otile = dst + base[r] + 128 * i * r;
-    const bool full = ng == 16;   // warp-uniform: position (gp + j) mod 16 by a mask
-    const bool on = gp < ng;
-    // rows in batches of 2 x kDeqRows: every load of a batch is issued before the first use, so a
-    // warp keeps kDeqRows code words and group parameters per lane in flight
-    for (int j0 = 0; j0 < r; j0 += 2 * kDeqRows) {
-      typename CodeWord<BITS>::T w[kDeqRows];
-      uint32_t par[kDeqRows];
-#pragma unroll
-      for (int u = 0; u < kDeqRows; ++u) {
-        const int j = j0 + 2 * u + lr;
-        if (on && j < r) {
-          const uint8_t* row = qtile + (long long)j * qrow;
-          w[u] = *reinterpret_cast<const typename CodeWord<BITS>::T*>(row + (BITS == 4 ? 4 : 8) * gp);
-          par[u] = *reinterpret_cast<const uint32_t*>(row + tl * BITS / 8 + 4 * (gp >> 2));
-        }
-      }
-#pragma unroll
-      for (int u = 0; u < kDeqRows; ++u) {
-        const int j = j0 + 2 * u + lr;
-        if (on && j < r) {
-          uint32_t c[8];
-          CodeWord<BITS>::unpack(w[u], c);
-          const __half2 ph = *reinterpret_cast<const __half2*>(&par[u]);
-          const float lo = __low2float(ph), st = __high2float(ph);
-          uint32_t o[4];
-#pragma unroll
-          for (int e = 0; e < 4; ++e) {   // lo + code * step in one fused rounding, then bf16
-            const __nv_bfloat162 v = __floats2bfloat162_rn(fmaf((float)c[2 * e], st, lo),
-                                                           fmaf((float)c[2 * e + 1], st, lo));
-            o[e] = *reinterpret_cast<const uint32_t*>(&v);
-          }
-          const int pos = full ? ((gp + j) & 15) : (gp + j) % ng;
-          *reinterpret_cast<uint4*>(otile + (long long)j * tl + 8 * pos) = make_uint4(o[0], o[1], o[2], o[3]);
-        }
-      }
-    }
-  }
-}
-
 }  // namespace
-
-size_t decode_q_expand_ws_bytes(const Shape& s, int num_sms) {
-  Shape s1 = s;
-  s1.L = 1;
-  const size_t dws = decode_ws_bytes(s1, num_sms);
-  const size_t coef = ((size_t)s.B * s.G * 2 * (size_t)s.cap * 2 + 255) & ~size_t(255);
-  const size_t cnt = ((size_t)s.B * (kMaxR + 1) * 4 + 255) & ~size_t(255);
-  const size_t base = ((size_t)s.B * (kMaxR + 2) * 8 + 255) & ~size_t(255);
-  return dws + coef + cnt + base;
-}
-
-bool decode_q_expand_supported(const Shape& s, int n_tail, int num_sms) {
-  Shape s1 = s;
-  s1.L = 1;
-  return s.dtype == VARRATE_BF16 && decode_mma_supported(s1, n_tail, num_sms) && s.B <= 65535;
-}
-
-int launch_decode_q_expand(const Shape& s, const varrate_qpacked& cache, const void* basis_k,
-                           const void* basis_v, const void* q, int layer, const void* tail_k,
-                           const void* tail_v, int n_tail, void* out, int32_t* dev_status, void* ws,
-                           int num_sms, cudaStream_t st) {
-  Shape s1 = s;
-  s1.L = 1;
-  char* w = static_cast<char*>(ws);
-  const size_t dws = decode_ws_bytes(s1, num_sms);
-  __nv_bfloat16* coef = reinterpret_cast<__nv_bfloat16*>(w + dws);
-  const size_t coef_b = ((size_t)s.B * s.G * 2 * (size_t)s.cap * 2 + 255) & ~size_t(255);
-  int32_t* cnt = reinterpret_cast<int32_t*>(w + dws + coef_b);
-  const size_t cnt_b = ((size_t)s.B * (kMaxR + 1) * 4 + 255) & ~size_t(255);
-  int64_t* base = reinterpret_cast<int64_t*>(w + dws + coef_b + cnt_b);
-  const dim3 grid(2 * s.G, s.B, kDeqSplit);
-  if (cache.bits == 4)
-    dequant_layer_kernel<4><<<grid, 256, 0, st>>>(cache.data, cache.qbase, cache.bucket_count, coef, cnt,
-                                                  base, dev_status, s, layer, cache.qcap_bytes);
-  else
-    dequant_layer_kernel<8><<<grid, 256, 0, st>>>(cache.data, cache.qbase, cache.bucket_count, coef, cnt,
-                                                  base, dev_status, s, layer, cache.qcap_bytes);
-  varrate_packed view = {};
-  view.coef = coef;
-  view.bucket_count = cnt;
-  view.bucket_base = base;
-  view.cap_elems = s.cap;
-  const size_t bstride = (size_t)layer * s.G * kHeadDim * kHeadDim;
-  const int rc = launch_decode(s1, view, static_cast<const __nv_bfloat16*>(basis_k) + bstride,
-                               static_cast<const __nv_bfloat16*>(basis_v) + bstride, q, 0, tail_k, tail_v,
-                               n_tail, out, dev_status, ws, num_sms, st);
-  return rc < 0 ? rc : rc + 1;
-}
 
 int launch_quantize(const Shape& s, const varrate_packed& in, const varrate_qpacked& out,
                     int32_t* dev_status, cudaStream_t st) {

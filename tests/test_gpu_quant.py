@@ -129,12 +129,12 @@ def test_quantize_bit_exact(name, bits):
                 np.testing.assert_array_equal(st[mask].view(np.uint16), want[2][mask].view(np.uint16))
 
 
-# workspace CALL_DECODE: the general kernels on x^ (fp32); CALL_DECODE_Q: the layer expanded to
-# bf16, then the fused tensor-core decode (beyond 256 tail tokens the general kernels again)
+# up to 256 tail tokens the fused kernel (codes dequantized in the ring, fp16 tiles) runs on either
+# workspace size; beyond that the general kernels on x^ (fp32)
 @pytest.mark.parametrize("bits,n_tail,which", [(4, 0, "DECODE"), (8, 0, "DECODE"), (4, 37, "DECODE"),
-                                               (4, 0, "DECODE_Q"), (8, 0, "DECODE_Q"),
-                                               (4, 37, "DECODE_Q"), (8, 256, "DECODE_Q"),
-                                               (4, 300, "DECODE_Q")])
+                                               (4, 0, "DECODE_Q"), (8, 37, "DECODE_Q"),
+                                               (8, 256, "DECODE"), (4, 300, "DECODE"),
+                                               (8, 300, "DECODE_Q")])
 @pytest.mark.parametrize("name", list(CASES))
 def test_decode_on_quantized_cache(name, bits, n_tail, which):
     wl, cfg, bk, bv, refs, packed, coefs, pairs = _setup(name)
