@@ -173,6 +173,62 @@ def test_decode_on_quantized_cache(name, bits, n_tail, which):
     print(f"{name} {bits}-bit ({which}): decode worst relative / absolute error {worst[0]:.3e} / {worst[1]:.3e}")
 
 
+@pytest.mark.parametrize("bits", [4, 8])
+def test_quantized_decode_deterministic_and_workspace_reuse(bits):
+    """Two fused calls on one workspace (garbage-filled first: beyond its header it is scratch) and a
+    call on a fresh zero-filled one give bit-identical outputs."""
+    wl, cfg, bk, bv, refs, packed, coefs, pairs = _setup("llama_ragged")
+    qp = V.QPackedCache.allocate(cfg, packed, bits)
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    V.check(V.varrate_quantize(cfg, packed, qp, status), "varrate_quantize")
+    q = synth.stack_decode_queries(wl, 1, 1)[0].cuda()
+    outs = []
+    ws = V.workspace(cfg, V.CALL_DECODE)
+    ws[33024:].fill_(0x5A)   # beyond the 33024-byte counter header
+    for w in (ws, ws, V.workspace(cfg, V.CALL_DECODE)):
+        out = torch.empty_like(q)
+        V.check(V.varrate_decode_attn_q(cfg, qp, bk.cuda(), bv.cuda(), q, 1, None, None, 0, out, status, w),
+                "varrate_decode_attn_q")
+        torch.cuda.synchronize()
+        assert int(status.item()) == V.OK
+        outs.append(out)
+    assert torch.equal(outs[0], outs[1]) and torch.equal(outs[0], outs[2])
+
+
+@pytest.mark.parametrize("bits", [4, 8])
+def test_quantized_decode_tail_only(bits):
+    """Empty coded set (the context is the exact window): the quantized streams hold only the
+    window's rank-d tile; with an exact tail the fused kernel's result is the oracle's."""
+    wl = synth.workload("llama1", n_kv_heads=2, n_ctx=32, window=32, batch=2)
+    k, v, qw, bk, bv = synth.stack_inputs(wl)
+    cfg = cfg_for(wl)
+    pairs = [(b, 0) for b in range(wl.batch)]
+    refs = {(b, 0): oracle_layer(wl, k, v, qw, bk, bv, b, 0) for b in range(wl.batch)}
+    packed, coefs = oracle_cache(wl, refs, cfg, pairs)
+    qp = V.QPackedCache.allocate(cfg, packed, bits)
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    V.check(V.varrate_quantize(cfg, packed, qp, status), "varrate_quantize")
+    gen = torch.Generator().manual_seed(3)
+    n_tail = 19
+    shape = (wl.batch, wl.n_kv_heads, n_tail, wl.head_dim)
+    tk = torch.randn(shape, generator=gen).to(torch.bfloat16)
+    tv = torch.randn(shape, generator=gen).to(torch.bfloat16)
+    q = synth.stack_decode_queries(wl, 0, 1)[0]
+    out = torch.empty_like(q, device="cuda")
+    V.check(V.varrate_decode_attn_q(cfg, qp, bk.cuda(), bv.cuda(), q.cuda(), 0, tk.cuda(), tv.cuda(), n_tail,
+                                    out, status, V.workspace(cfg, V.CALL_DECODE)), "varrate_decode_attn_q")
+    torch.cuda.synchronize()
+    assert int(status.item()) == V.OK
+    got = f64(out)
+    for b in range(wl.batch):
+        ref = refs[(b, 0)]
+        deq = [[O.quantize_coefficients(coefs[(b, 0)][g, kv], ref["ranks"], ref["count"], ref["pos"], bits)[3]
+                for g in range(wl.n_kv_heads)] for kv in range(2)]
+        want = O.decode_coef(f64(q[b]), np.stack(deq[0]).astype(np.float64), np.stack(deq[1]).astype(np.float64),
+                             ref["ranks"], f64(bk[0]), f64(bv[0]), f64(tk[b]), f64(tv[b]))
+        assert decode_close(got[b], want, cfg), (b, decode_errors(got[b], want))
+
+
 def test_quantized_round_trip_bound_at_full_size():
     """llama32 layer call (8 sequences x 8 KV heads x N = 32768, GPU encode): every quantized group
     reproduces the stored coefficients within half a step plus the fp16 rounding of its offset
@@ -227,7 +283,7 @@ def test_quantized_round_trip_bound_at_full_size():
 
 def test_quantized_decode_full_size():
     """llama32 layer call (8 sequences x 8 KV heads x N = 32768, GPU encode), 4-bit, through the
-    fused path (layer expanded to bf16, then the tensor-core decode) in the launch configuration
+    fused kernel (codes dequantized in the ring, fp16 tensor-core tiles) in the launch configuration
     bench.py times: one sampled sequence against the oracle's decode on its own quantization of the
     same stored coefficients, and a score-blind output failing the same bar."""
     from gpu_helpers import uniform_weight_output, unpack
