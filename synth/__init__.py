@@ -21,9 +21,11 @@ Workloads (stand-ins for the paper's LongBench / NIAH prompts, whose models and 
 Data model for one (sequence, layer, KV head, K-or-V) stream of N tokens:
     X = (Z * sigma * scale) @ F^T + noise_std * E,   Z, E ~ N(0, 1) i.i.d. [N, d]
 where F is a seeded orthonormal d x d frame and ``scale`` makes the mean per-entry variance 1.
-The per-head basis handed to the codec is F^T (row j = frame direction j, ordered by decreasing
-sigma): the basis the paper's offline PCA (Sec. 3.1, "Shared basis") converges to on this
-distribution. Queries are N(0, 1).
+The per-head basis handed to the codec stands in for the paper's offline calibration (Sec. 3.1,
+"Shared basis": the leading right singular vectors of calibration activations): the right singular
+vectors, in fp64 (the eigenvectors of the Gram matrix), of a separate draw of CALIB_TOKENS tokens
+from the same distribution (its own seeds), rows ordered by decreasing singular value, each row's
+sign fixed so that its largest component is positive. Queries are N(0, 1).
 
 Seeds are a pure function of (workload id, sequence, layer, head, stream kind); the same call on
 the same device always returns the same tensor. CPU draws use torch's CPU generator, CUDA draws
@@ -32,6 +34,7 @@ that compares two paths always feeds both the same drawn tensor.
 """
 from __future__ import annotations
 
+import functools
 import math
 from dataclasses import dataclass, field, replace
 
@@ -42,7 +45,8 @@ __all__ = ["Workload", "WORKLOADS", "workload", "frames", "bases", "layer_kv", "
            "decode_queries", "outlier_tokens", "seed_of"]
 
 _KIND = {"k": 0, "v": 1, "qwin": 2, "qdec": 3, "outlier": 4, "frame": 5, "noise_k": 6,
-         "noise_v": 7}
+         "noise_v": 7, "calib": 8}
+CALIB_TOKENS = 2048   # tokens of the separate calibration draw the bases are fitted to
 
 
 @dataclass(frozen=True)
@@ -125,9 +129,8 @@ def _scale(wl: Workload) -> float:
     return math.sqrt((1.0 - wl.noise_std ** 2) * wl.head_dim / float(np.sum(sig ** 2)))
 
 
-def frames(wl: Workload, layer: int) -> np.ndarray:
-    """Orthonormal frames F [G][2][d][d] (fp64) for one layer: QR of a seeded Gaussian, with the
-    diagonal of R made positive so the frame is unique for the seed."""
+@functools.lru_cache(maxsize=256)
+def _frames(wl: Workload, layer: int) -> np.ndarray:
     d = wl.head_dim
     out = np.empty((wl.n_kv_heads, 2, d, d))
     for g in range(wl.n_kv_heads):
@@ -137,14 +140,40 @@ def frames(wl: Workload, layer: int) -> np.ndarray:
             q, r = np.linalg.qr(a)
             q = q * np.sign(np.diag(r))[None, :]
             out[g, kv] = q
+    out.setflags(write=False)
     return out
 
 
+def frames(wl: Workload, layer: int) -> np.ndarray:
+    """Orthonormal frames F [G][2][d][d] (fp64) for one layer: QR of a seeded Gaussian, with the
+    diagonal of R made positive so the frame is unique for the seed."""
+    return np.array(_frames(wl, layer))
+
+
+@functools.lru_cache(maxsize=256)
+def _bases(wl: Workload, layer: int) -> tuple[np.ndarray, np.ndarray]:
+    d, n, G = wl.head_dim, CALIB_TOKENS, wl.n_kv_heads
+    f = torch.from_numpy(frames(wl, layer).reshape(2 * G, d, d))   # stream 2 g + kv
+    sig = torch.from_numpy(spectrum(wl) * _scale(wl))
+    zs = torch.randn((2, 2 * G, n, d), generator=_gen(seed_of(wl, "calib", 0, layer), "cpu"),
+                     dtype=torch.float32).double()
+    x = (zs[0] * sig) @ f.transpose(1, 2)
+    if wl.noise_std > 0:
+        x += wl.noise_std * zs[1]
+    # right singular vectors of each draw = eigenvectors of its Gram matrix, by decreasing eigenvalue
+    vt = np.linalg.eigh((x.transpose(1, 2) @ x).numpy())[1][:, :, ::-1].transpose(0, 2, 1)
+    lead = np.take_along_axis(vt, np.argmax(np.abs(vt), axis=2)[:, :, None], axis=2)
+    vt = vt * np.sign(lead)
+    out = np.ascontiguousarray(vt.reshape(G, 2, d, d).transpose(1, 0, 2, 3))
+    out.setflags(write=False)
+    return out[0], out[1]
+
+
 def bases(wl: Workload, layer: int) -> tuple[np.ndarray, np.ndarray]:
-    """Per-head bases U_K, U_V [G][d][d] (fp64), row j = basis vector j (frame column j)."""
-    f = frames(wl, layer)
-    return (np.ascontiguousarray(np.transpose(f[:, 0], (0, 2, 1))),
-            np.ascontiguousarray(np.transpose(f[:, 1], (0, 2, 1))))
+    """Per-head bases U_K, U_V [G][d][d] (fp64), row j = basis vector j: the right singular vectors
+    of a separate calibration draw (module docstring)."""
+    uk, uv = _bases(wl, layer)
+    return np.array(uk), np.array(uv)
 
 
 def torch_dtype(wl: Workload) -> torch.dtype:
