@@ -310,6 +310,15 @@ varrate_status varrate_decode_attn_noalloc(const varrate_config* cfg, const varr
                                            int32_t n_tail, void* out, int32_t* dev_status,
                                            void* stream);
 
+/* Self-test of the device-side failure path (no counterpart in the paper). Every TMA, tcgen05 and
+ * bulk-copy wait in the library is a bounded loop of mbarrier polls; one that gives up raises
+ * VARRATE_ERR_TIMEOUT in *dev_status and the kernel returns, leaving the context usable. This call
+ * runs one block that waits on an mbarrier phase nothing completes, for 1 <= polls <= 2^24 polls, so
+ * it always raises VARRATE_ERR_TIMEOUT in *dev_status (an int32 in device memory, 4-byte aligned);
+ * no copy is in flight, so nothing can fault. VARRATE_ERR_ARG for a NULL or misaligned status word
+ * or polls out of range. */
+varrate_status varrate_selftest_wait_timeout(int32_t* dev_status, uint32_t polls, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -104,6 +104,7 @@ _SIGS = {
                                                      _c_void_p, _c_void_p, ctypes.c_int32,
                                                      _c_void_p, _c_void_p, ctypes.c_int32,
                                                      _c_void_p, _c_void_p, _c_void_p]),
+    "varrate_selftest_wait_timeout": (ctypes.c_int32, [_c_void_p, ctypes.c_uint32, _c_void_p]),
 }
 
 EXPORTED = tuple(_SIGS)
@@ -225,6 +226,10 @@ def varrate_decode_attn_noalloc(cfg, packed, basis_k, basis_v, q, layer, tail_k,
                                              _ptr(basis_k), _ptr(basis_v), _ptr(q), layer,
                                              _ptr(tail_k), _ptr(tail_v), n_tail, _ptr(out),
                                              _ptr(dev_status), _stream(stream))
+
+
+def varrate_selftest_wait_timeout(dev_status, polls, stream=None) -> int:
+    return lib().varrate_selftest_wait_timeout(_ptr(dev_status), polls, _stream(stream))
 
 
 def varrate_decode_window(cfg, packed, basis_k, basis_v, q, n_q, layer, tail_k, tail_v, n_tail, out,

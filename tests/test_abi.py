@@ -212,3 +212,15 @@ def test_packed_cache_and_workspace_helpers(vlib):
     ws = vlib.workspace(cfg, vlib.CALL_DECODE, "cpu")
     assert ws.numel() >= vlib.varrate_workspace_bytes(cfg, vlib.CALL_DECODE)
     assert int(vlib.torch.count_nonzero(ws)) == 0
+
+
+def test_selftest_wait_rejects_bad_arguments_on_host(vlib):
+    """The bounded-wait self-test validates its arguments before anything is launched."""
+    import ctypes
+    buf = ctypes.create_string_buffer(16)
+    base = ctypes.addressof(buf)
+    aligned = base + ((-base) % 4)
+    assert vlib.lib().varrate_selftest_wait_timeout(None, 8, None) == vlib.ERR_ARG
+    assert vlib.lib().varrate_selftest_wait_timeout(ctypes.c_void_p(aligned), 0, None) == vlib.ERR_ARG
+    assert vlib.lib().varrate_selftest_wait_timeout(ctypes.c_void_p(aligned), (1 << 24) + 1, None) == vlib.ERR_ARG
+    assert vlib.lib().varrate_selftest_wait_timeout(ctypes.c_void_p(aligned + 1), 8, None) == vlib.ERR_ARG
