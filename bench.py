@@ -602,6 +602,48 @@ def sweep_quant(V, wl, dev, peak, stream, decode_steps, bits_list=(4, 8)):
     return res
 
 
+def sweep_anchor_search(V, wl, dev, stream, stride=16, c=4):
+    """Joint codec: the nearest-anchor search (Sec. 3.1, Eq. 2) over every (sequence, layer) of a
+    Llama-shaped stack (D = 2 G d = 2048 joint coordinates, N / stride anchors). Algorithmic work
+    per (sequence, layer): 2 N n_a D flops for the dot products (tensor cores, bf16 -> fp32) and
+    one read of K and V (2 G N d bf16) for the norms and the anchor copy."""
+    with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+        tf_peak = float(json.load(f)["bf16_tflops"])
+    cfg = V.make_config(wl.n_layers, wl.n_kv_heads, wl.group, wl.n_ctx, batch=wl.batch,
+                        window=wl.window, dtype=V.BF16)
+    k, v, _, _, _ = synth.stack_inputs(wl, device=dev)
+    units = wl.batch * wl.n_layers
+    n_a = (wl.n_ctx + stride - 1) // stride
+    D = 2 * wl.n_kv_heads * wl.head_dim
+    idx = torch.empty((wl.batch, wl.n_layers, wl.n_ctx, c), dtype=torch.int32, device=dev)
+    dist = torch.empty((wl.batch, wl.n_layers, wl.n_ctx, c), dtype=torch.float32, device=dev)
+    ws = torch.zeros(V.varrate_anchor_search_ws_bytes(cfg, stride), dtype=torch.uint8, device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    times = []
+    for i in range(6):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        V.check(V.varrate_anchor_search(cfg, k, v, stride, c, idx, dist, status, ws, stream),
+                "varrate_anchor_search")
+        e1.record(stream)
+        torch.cuda.synchronize()
+        if i >= 2:
+            times.append(e0.elapsed_time(e1))
+    ms = statistics.median(times)
+    flops = 2.0 * wl.n_ctx * n_a * D * units
+    tflops = flops / (ms * 1e-3) / 1e12
+    res = {"workload": workload_desc(wl), "stride": stride, "c": c, "anchors": n_a, "joint_dim": D,
+           "ms_per_layer": round(ms / units, 4), "ms_per_call": round(ms, 3),
+           "tflops": round(tflops, 1), "frac_of_bf16_peak": round(tflops / tf_peak, 4),
+           "status": V.status_string(int(status.item())),
+           "kernels": "per call: a norm and anchor-copy pass over K and V, then the tcgen05 search "
+                      "(M = 128 tokens x N = 256 anchors, K = D, TMA-fed); the time and the TFLOP/s "
+                      "cover both"}
+    del k, v, idx, dist, ws
+    torch.cuda.empty_cache()
+    return res
+
+
 def run_sweep(args, peak):
     """The other seeded configurations, each with its own encode and decode numbers."""
     from paper_2607_15498_gb300 import varrate as V
@@ -621,6 +663,8 @@ def run_sweep(args, peak):
                                n_window=32, n_decode=wl.decode_steps)
     out["llama32_quantized"] = sweep_quant(V, synth.workload("llama32", n_layers=4), dev, peak,
                                            stream, decode_steps=32)
+    out["joint_anchor_search"] = sweep_anchor_search(V, synth.workload("llama32", n_layers=4, batch=2),
+                                                     dev, stream)
     return out
 
 

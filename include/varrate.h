@@ -319,6 +319,30 @@ varrate_status varrate_decode_attn_noalloc(const varrate_config* cfg, const varr
  * or polls out of range. */
 varrate_status varrate_selftest_wait_timeout(int32_t* dev_status, uint32_t polls, void* stream);
 
+/* Joint codec, nearest anchors (Sec. 3.1, Eq. 1-2) — the search step of the paper's residual codec.
+ * For one (sequence, layer) the joint per-token vector stacks every KV head's key and value,
+ *   z_t = [k_t of heads 0..G-1 ; v_t of heads 0..G-1]  (D = 2 G d),
+ * the anchors are the tokens a * stride (a = 0 .. n_a - 1, n_a = ceil(N / stride)), and for every
+ * token t this call lists the c anchors nearest z_t in squared Euclidean distance,
+ *   dist(t, a) = max(0, |z_t|^2 + |z_a|^2 - 2 z_t . z_a),
+ * with the bf16 products exact and the sums in fp32 (tensor cores for the dot products), ordered by
+ * (distance, a). Tokens that are anchors are listed too (their own anchor comes first).
+ *   k, v      [B][L][G][N][d] bf16 (the encode inputs)
+ *   stride    1 <= stride <= N;  c: 1 <= c <= 8
+ *   idx_out   [B][L][N][c] int32 anchor numbers (the anchor token is a * stride); -1 past n_a
+ *   dist_out  [B][L][N][c] fp32 squared distances, +inf past n_a; may be NULL
+ *   ws        at least varrate_anchor_search_ws_bytes(cfg, stride) bytes of scratch (the anchors
+ *             copied densely, their norms and the token norms), written before it is read.
+ * Limits: dtype VARRATE_BF16, batch * n_layers <= 65535, n_kv_heads <= 64 (VARRATE_ERR_UNSUPPORTED
+ * otherwise). Only n_layers, n_kv_heads, head_dim, n_ctx, batch and dtype of cfg are used (the
+ * rest must still pass varrate_check_config). Two kernels run: one pass over K and V for the
+ * norms and the anchor copy, then the tensor-core search. A wait that gives up raises
+ * VARRATE_ERR_TIMEOUT in *dev_status and leaves the outputs of that tile unwritten. */
+size_t varrate_anchor_search_ws_bytes(const varrate_config* cfg, int32_t stride);
+varrate_status varrate_anchor_search(const varrate_config* cfg, const void* k, const void* v,
+                                     int32_t stride, int32_t c, int32_t* idx_out, float* dist_out,
+                                     int32_t* dev_status, void* ws, size_t ws_bytes, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -75,26 +75,29 @@ def exact_mask(n_ctx: int, stride: int, window: int) -> np.ndarray:
 
 # ------------------------------------------------------- nearest anchors (Sec. 3.1, Eq. 2)
 
-def nearest_anchors(z: np.ndarray, stride: int, c: int):
+def nearest_anchors(z: np.ndarray, stride: int, c: int, rows=None):
     """The c anchors nearest every token in squared Euclidean distance over the joint vector.
 
     Returns (idx int64 [N][c]: anchor numbers a, the anchor token being z[a * stride],
     dist fp64 [N][c]: the squared distances), each row ordered by (distance, anchor number).
-    Rows of tokens that are themselves anchors are included (their nearest anchor is themselves)."""
+    Rows of tokens that are themselves anchors are included (their nearest anchor is themselves).
+    With ``rows`` (token indices) only those tokens are searched and the results have one row per
+    listed token, in the given order."""
     z = np.asarray(z, dtype=np.float64)
     N = z.shape[0]
     pos = anchor_positions(N, stride)
     anchors = z[pos]
     n_a = pos.size
-    idx = np.full((N, c), -1, dtype=np.int64)
-    dist = np.full((N, c), np.inf)
-    for t in range(N):
+    tokens = np.arange(N) if rows is None else np.asarray(rows, dtype=np.int64)
+    idx = np.full((tokens.size, c), -1, dtype=np.int64)
+    dist = np.full((tokens.size, c), np.inf)
+    for i, t in enumerate(tokens):
         diff = anchors - z[t]
         d2 = np.einsum("ad,ad->a", diff, diff)
         order = np.lexsort((np.arange(n_a), d2))       # by distance, then anchor number
         take = order[:min(c, n_a)]
-        idx[t, :take.size] = take
-        dist[t, :take.size] = d2[take]
+        idx[i, :take.size] = take
+        dist[i, :take.size] = d2[take]
     return idx, dist
 
 

@@ -329,4 +329,27 @@ varrate_status varrate_decode_attn_q(const varrate_config* cfg, const varrate_qp
   return launched();
 }
 
+size_t varrate_anchor_search_ws_bytes(const varrate_config* cfg, int32_t stride) {
+  if (check(cfg) != VARRATE_OK || stride < 1 || stride > cfg->n_ctx) return 0;
+  return vr::anchor_search_ws_bytes(make_shape(cfg, cap_elems(cfg)), stride);
+}
+
+varrate_status varrate_anchor_search(const varrate_config* cfg, const void* k, const void* v,
+                                     int32_t stride, int32_t c, int32_t* idx_out, float* dist_out,
+                                     int32_t* dev_status, void* ws, size_t ws_bytes_, void* stream) {
+  varrate_status st = check(cfg);
+  if (st != VARRATE_OK) return st;
+  if (cfg->dtype != VARRATE_BF16) return VARRATE_ERR_UNSUPPORTED;
+  if (!k || !v || !idx_out || stride < 1 || stride > cfg->n_ctx || c < 1) return VARRATE_ERR_ARG;
+  if (!aligned16({k, v, idx_out, dist_out, dev_status, ws})) return VARRATE_ERR_ARG;
+  const Shape s = make_shape(cfg, cap_elems(cfg));
+  if (!vr::anchor_search_supported(s, stride, c)) return VARRATE_ERR_UNSUPPORTED;
+  const size_t need = vr::anchor_search_ws_bytes(s, stride);
+  if (ws_bytes_ < need || ws == nullptr) return VARRATE_ERR_WORKSPACE;
+  if (vr::launch_anchor_search(s, k, v, stride, c, idx_out, dist_out, dev_status, ws,
+                               (cudaStream_t)stream) < 0)
+    return VARRATE_ERR_CUDA;
+  return launched();
+}
+
 }  // extern "C"

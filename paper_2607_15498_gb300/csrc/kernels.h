@@ -95,4 +95,12 @@ int launch_decode_q(const Shape& s, const varrate_qpacked& cache, const void* ba
                     const void* basis_v, const void* q, int layer, const void* tail_k,
                     const void* tail_v, int n_tail, void* out, void* ws, int num_sms, cudaStream_t st);
 
+// ---- joint codec: nearest-anchor search (anchor_search.cu)
+int anchor_count(int64_t N, int stride);
+int anchor_count_padded(int64_t N, int stride);   // rounded up to the 256-anchor MMA tile
+size_t anchor_search_ws_bytes(const Shape& s, int stride);
+bool anchor_search_supported(const Shape& s, int stride, int c);
+int launch_anchor_search(const Shape& s, const void* k, const void* v, int stride, int c, int32_t* idx_out,
+                         float* dist_out, int32_t* dev_status, void* ws, cudaStream_t st);
+
 }  // namespace vr

@@ -105,6 +105,10 @@ _SIGS = {
                                                      _c_void_p, _c_void_p, ctypes.c_int32,
                                                      _c_void_p, _c_void_p, _c_void_p]),
     "varrate_selftest_wait_timeout": (ctypes.c_int32, [_c_void_p, ctypes.c_uint32, _c_void_p]),
+    "varrate_anchor_search_ws_bytes": (ctypes.c_size_t, [ctypes.POINTER(varrate_config), ctypes.c_int32]),
+    "varrate_anchor_search": (ctypes.c_int32, [ctypes.POINTER(varrate_config), _c_void_p, _c_void_p,
+                                               ctypes.c_int32, ctypes.c_int32, _c_void_p, _c_void_p,
+                                               _c_void_p, _c_void_p, ctypes.c_size_t, _c_void_p]),
 }
 
 EXPORTED = tuple(_SIGS)
@@ -230,6 +234,16 @@ def varrate_decode_attn_noalloc(cfg, packed, basis_k, basis_v, q, layer, tail_k,
 
 def varrate_selftest_wait_timeout(dev_status, polls, stream=None) -> int:
     return lib().varrate_selftest_wait_timeout(_ptr(dev_status), polls, _stream(stream))
+
+
+def varrate_anchor_search_ws_bytes(cfg: varrate_config, stride: int) -> int:
+    return lib().varrate_anchor_search_ws_bytes(ctypes.byref(cfg), stride)
+
+
+def varrate_anchor_search(cfg, k, v, stride, c, idx_out, dist_out, dev_status, ws, stream=None) -> int:
+    return lib().varrate_anchor_search(ctypes.byref(cfg), _ptr(k), _ptr(v), stride, c, _ptr(idx_out),
+                                       _ptr(dist_out), _ptr(dev_status), _ptr(ws), _nbytes(ws),
+                                       _stream(stream))
 
 
 def varrate_decode_window(cfg, packed, basis_k, basis_v, q, n_q, layer, tail_k, tail_v, n_tail, out,

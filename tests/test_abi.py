@@ -224,3 +224,32 @@ def test_selftest_wait_rejects_bad_arguments_on_host(vlib):
     assert vlib.lib().varrate_selftest_wait_timeout(ctypes.c_void_p(aligned), 0, None) == vlib.ERR_ARG
     assert vlib.lib().varrate_selftest_wait_timeout(ctypes.c_void_p(aligned), (1 << 24) + 1, None) == vlib.ERR_ARG
     assert vlib.lib().varrate_selftest_wait_timeout(ctypes.c_void_p(aligned + 1), 8, None) == vlib.ERR_ARG
+
+
+def test_anchor_search_host_checks(vlib):
+    """Workspace size of the nearest-anchor search and the argument checks made before any launch:
+    anchors padded to 256 (ceil(1000 / 16) = 63 -> 256), 3 sequences x 2 layers, G = 8:
+    anchors 6 * 2 * 8 * 256 * 128 * 2 B, their norms 6 * 256 * 4 B, token norms 6 * 1000 * 4 B,
+    each rounded up to 256 B."""
+    L = vlib.lib()
+    cfg = vlib.make_config(2, 8, 4, 1000, batch=3, dtype=vlib.BF16)
+    assert vlib.varrate_anchor_search_ws_bytes(cfg, 16) == 6291456 + 6144 + 24064
+    assert vlib.varrate_anchor_search_ws_bytes(cfg, 0) == 0
+    assert vlib.varrate_anchor_search_ws_bytes(cfg, 1001) == 0
+    need = vlib.varrate_anchor_search_ws_bytes(cfg, 16)
+
+    def call(c=cfg, k=A, v=A, stride=16, n=4, idx=A, dist=A, ws=A, nbytes=need):
+        return L.varrate_anchor_search(vlib.ctypes.byref(c), k, v, stride, n, idx, dist, None, ws,
+                                       nbytes, None)
+    assert call(k=None) == vlib.ERR_ARG
+    assert call(idx=None) == vlib.ERR_ARG
+    assert call(stride=0) == vlib.ERR_ARG
+    assert call(stride=1001) == vlib.ERR_ARG
+    assert call(n=0) == vlib.ERR_ARG
+    assert call(n=9) == vlib.ERR_UNSUPPORTED
+    assert call(v=A + 8) == vlib.ERR_ARG
+    assert call(dist=A + 4) == vlib.ERR_ARG
+    assert call(nbytes=need - 1) == vlib.ERR_WORKSPACE
+    assert call(ws=None) == vlib.ERR_WORKSPACE
+    f32 = vlib.make_config(2, 8, 4, 1000, batch=3, dtype=vlib.F32)
+    assert call(c=f32) == vlib.ERR_UNSUPPORTED

@@ -124,6 +124,10 @@ def test_nearest_anchors_scipy_cdist():
     ref = np.argsort(d2, axis=1, kind="stable")[:, :c]
     np.testing.assert_array_equal(idx, ref)
     np.testing.assert_allclose(dist, np.take_along_axis(d2, ref, axis=1), rtol=1e-12, atol=1e-12)
+    rows = np.array([299, 0, 17, 150])
+    ri, rd = J.nearest_anchors(z, stride, c, rows=rows)
+    np.testing.assert_array_equal(ri, ref[rows])
+    np.testing.assert_array_equal(rd, dist[rows])
 
 
 def test_anchor_tokens_pick_themselves_and_ties_take_the_lower_index():
