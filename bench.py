@@ -813,6 +813,9 @@ def main():
                     help="issue the headline decode calls from the host instead of replaying a graph")
     ap.add_argument("--layers", type=int, default=None, help="override the layer count (profiling)")
     ap.add_argument("--batch", type=int, default=None, help="override the sequence count (profiling)")
+    ap.add_argument("--anchor-search-only", action="store_true",
+                    help="time only the joint codec's nearest-anchor search on the workload and print "
+                         "its JSON (profiling)")
     args = ap.parse_args()
     wl = synth.workload(args.workload)
     if args.layers is not None:
@@ -870,6 +873,12 @@ def main():
         torch.cuda.set_device(local)
     else:
         torch.cuda.set_device(0)
+    if args.anchor_search_only:
+        from paper_2607_15498_gb300 import varrate as V
+        if rank == 0:
+            print(json.dumps(sweep_anchor_search(V, wl, torch.device("cuda", torch.cuda.current_device()),
+                                                 torch.cuda.current_stream())))
+        return
     r = run_ours(args, wl, rank, world)
     K = args.steps
     total_s = r["total_ms"] * 1e-3
