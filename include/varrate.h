@@ -343,6 +343,21 @@ varrate_status varrate_anchor_search(const varrate_config* cfg, const void* k, c
                                      int32_t stride, int32_t c, int32_t* idx_out, float* dist_out,
                                      int32_t* dev_status, void* ws, size_t ws_bytes, void* stream);
 
+/* Joint codec, residuals (Sec. 3.1, Eq. 2; the third step of Algorithm 1): for every token t,
+ *   e_t = z_t - mean of the anchors z_{a * stride} listed for t,
+ * with z_t the joint vector of varrate_anchor_search. Arithmetic: the listed anchors' bf16 values
+ * summed in list order in fp32, divided (IEEE) by their count, subtracted from z_t in fp32,
+ * rounded to bf16.
+ *   k, v    [B][L][G][N][d] bf16
+ *   idx     [B][L][N][c] int32 anchor lists (e.g. from varrate_anchor_search); entries -1 are skipped
+ *   e_out   [B][L][N][2 G d] bf16, in the joint order (head g's key at g d, its value at G d + g d)
+ * A list with an entry outside [-1, n_a) or no valid entry raises VARRATE_ERR_CORRUPT in *dev_status
+ * and leaves that token's row unwritten. Limits: dtype VARRATE_BF16, 1 <= stride <= N,
+ * 1 <= c <= 8, batch * n_layers <= 65535. One kernel, no workspace. */
+varrate_status varrate_anchor_residual(const varrate_config* cfg, const void* k, const void* v,
+                                       int32_t stride, int32_t c, const int32_t* idx, void* e_out,
+                                       int32_t* dev_status, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

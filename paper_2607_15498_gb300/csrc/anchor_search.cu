@@ -18,6 +18,8 @@
 //                         8 smallest (distance, anchor) pairs in registers, in lexicographic order;
 //                         the two epilogue groups (alternate anchor tiles) merge their lists at the
 //                         end and the first c pairs are stored.
+// A third kernel, anchor_residual_kernel, forms the residuals e_t = z_t - z_bar_t of Eq. 2 from the
+// lists (Algorithm 1, third step).
 // Warp roles of the search kernel: one TMA producer warp, one MMA-issuing warp, eight epilogue
 // warps (lane quarter = warp % 4). Every mbarrier wait is bounded; a timeout raises
 // VARRATE_ERR_TIMEOUT.
@@ -249,6 +251,56 @@ anchor_search_tc_kernel(const __grid_constant__ CUtensorMap tk, const __grid_con
 
 size_t search_smem_bytes() { return 1024 + (size_t)AS_ST * AS_SBYTES + sizeof(AsSmem); }
 
+// ------------------------------------------------------------------------------ residual
+// Eq. 2: e_t = z_t - mean of the anchors listed for t. grid (ceil(N / 8), B * L), 256 threads: warp w
+// takes token blockIdx.x * 8 + w; lane l owns coordinates 4 l .. 4 l + 3 of every head row. The
+// listed anchors are summed in list order in fp32 (bf16 values are exact in fp32), divided by
+// their count (IEEE division), subtracted from z_t and rounded to bf16.
+__global__ void __launch_bounds__(256)
+anchor_residual_kernel(const __nv_bfloat16* __restrict__ k, const __nv_bfloat16* __restrict__ v,
+                       const int32_t* __restrict__ idx, __nv_bfloat16* __restrict__ e,
+                       int32_t* __restrict__ dev_status, int G, int64_t N, int stride, int c, int n_a) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t bl = blockIdx.y;
+  const int64_t t = (int64_t)blockIdx.x * 8 + warp;
+  if (t >= N) return;
+  int ai[AS_LIST];
+  int m = 0;
+  bool bad = false;
+#pragma unroll
+  for (int s = 0; s < AS_LIST; ++s) {
+    ai[s] = s < c ? __ldg(idx + (bl * N + t) * c + s) : -1;
+    if (ai[s] >= n_a || ai[s] < -1) bad = true;
+    if (ai[s] >= 0) ++m;
+  }
+  if (bad || m == 0) {                               // warp-uniform: every lane read the same list
+    if (lane == 0) raise_status(dev_status, VARRATE_ERR_CORRUPT);
+    return;
+  }
+  const float fm = (float)m;
+  for (int kvg = 0; kvg < 2 * G; ++kvg) {
+    const int kv = kvg >= G, g = kvg - kv * G;
+    const __nv_bfloat16* base = (kv ? v : k) + (bl * G + g) * N * kHeadDim;
+    const uint2 zu = __ldg(reinterpret_cast<const uint2*>(base + t * kHeadDim) + lane);
+    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+    for (int s = 0; s < AS_LIST; ++s) {
+      if (ai[s] < 0) continue;
+      const uint2 u = __ldg(reinterpret_cast<const uint2*>(base + (int64_t)ai[s] * stride * kHeadDim) + lane);
+      acc[0] += __uint_as_float(u.x << 16);
+      acc[1] += __uint_as_float(u.x & 0xffff0000u);
+      acc[2] += __uint_as_float(u.y << 16);
+      acc[3] += __uint_as_float(u.y & 0xffff0000u);
+    }
+    const float z0 = __uint_as_float(zu.x << 16), z1 = __uint_as_float(zu.x & 0xffff0000u);
+    const float z2 = __uint_as_float(zu.y << 16), z3 = __uint_as_float(zu.y & 0xffff0000u);
+    uint2 o;
+    o.x = pack_bf16(__fsub_rn(z0, __fdiv_rn(acc[0], fm)), __fsub_rn(z1, __fdiv_rn(acc[1], fm)));
+    o.y = pack_bf16(__fsub_rn(z2, __fdiv_rn(acc[2], fm)), __fsub_rn(z3, __fdiv_rn(acc[3], fm)));
+    reinterpret_cast<uint2*>(e + ((bl * N + t) * 2 * G + kvg) * kHeadDim)[lane] = o;
+  }
+}
+
 }  // namespace
 
 bool make_tmap_rows_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint32_t box_rows);
@@ -263,6 +315,19 @@ size_t anchor_search_ws_bytes(const Shape& s, int stride) {
   const size_t bl = (size_t)s.B * s.L;
   auto a256 = [](size_t x) { return (x + 255) & ~size_t(255); };
   return a256(bl * 2 * s.G * n_ap * kHeadDim * 2) + a256(bl * n_ap * 4) + a256(bl * (size_t)s.N * 4);
+}
+
+bool anchor_residual_supported(const Shape& s, int stride, int c) {
+  return s.dtype == VARRATE_BF16 && stride >= 1 && stride <= s.N && c >= 1 && c <= AS_LIST &&
+         (int64_t)s.B * s.L <= 65535;
+}
+
+int launch_anchor_residual(const Shape& s, const void* k, const void* v, int stride, int c,
+                           const int32_t* idx, void* e_out, int32_t* dev_status, cudaStream_t st) {
+  anchor_residual_kernel<<<dim3((unsigned)((s.N + 7) / 8), (unsigned)((size_t)s.B * s.L)), 256, 0, st>>>(
+      (const __nv_bfloat16*)k, (const __nv_bfloat16*)v, idx, (__nv_bfloat16*)e_out, dev_status, s.G, s.N,
+      stride, c, anchor_count(s.N, stride));
+  return 1;
 }
 
 bool anchor_search_supported(const Shape& s, int stride, int c) {

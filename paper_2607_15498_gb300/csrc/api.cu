@@ -352,4 +352,18 @@ varrate_status varrate_anchor_search(const varrate_config* cfg, const void* k, c
   return launched();
 }
 
+varrate_status varrate_anchor_residual(const varrate_config* cfg, const void* k, const void* v,
+                                       int32_t stride, int32_t c, const int32_t* idx, void* e_out,
+                                       int32_t* dev_status, void* stream) {
+  varrate_status st = check(cfg);
+  if (st != VARRATE_OK) return st;
+  if (cfg->dtype != VARRATE_BF16) return VARRATE_ERR_UNSUPPORTED;
+  if (!k || !v || !idx || !e_out || stride < 1 || stride > cfg->n_ctx || c < 1) return VARRATE_ERR_ARG;
+  if (!aligned16({k, v, idx, e_out, dev_status})) return VARRATE_ERR_ARG;
+  const Shape s = make_shape(cfg, cap_elems(cfg));
+  if (!vr::anchor_residual_supported(s, stride, c)) return VARRATE_ERR_UNSUPPORTED;
+  vr::launch_anchor_residual(s, k, v, stride, c, idx, e_out, dev_status, (cudaStream_t)stream);
+  return launched();
+}
+
 }  // extern "C"

@@ -102,5 +102,8 @@ size_t anchor_search_ws_bytes(const Shape& s, int stride);
 bool anchor_search_supported(const Shape& s, int stride, int c);
 int launch_anchor_search(const Shape& s, const void* k, const void* v, int stride, int c, int32_t* idx_out,
                          float* dist_out, int32_t* dev_status, void* ws, cudaStream_t st);
+bool anchor_residual_supported(const Shape& s, int stride, int c);
+int launch_anchor_residual(const Shape& s, const void* k, const void* v, int stride, int c,
+                           const int32_t* idx, void* e_out, int32_t* dev_status, cudaStream_t st);
 
 }  // namespace vr

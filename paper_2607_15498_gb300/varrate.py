@@ -109,6 +109,9 @@ _SIGS = {
     "varrate_anchor_search": (ctypes.c_int32, [ctypes.POINTER(varrate_config), _c_void_p, _c_void_p,
                                                ctypes.c_int32, ctypes.c_int32, _c_void_p, _c_void_p,
                                                _c_void_p, _c_void_p, ctypes.c_size_t, _c_void_p]),
+    "varrate_anchor_residual": (ctypes.c_int32, [ctypes.POINTER(varrate_config), _c_void_p, _c_void_p,
+                                                 ctypes.c_int32, ctypes.c_int32, _c_void_p, _c_void_p,
+                                                 _c_void_p, _c_void_p]),
 }
 
 EXPORTED = tuple(_SIGS)
@@ -244,6 +247,11 @@ def varrate_anchor_search(cfg, k, v, stride, c, idx_out, dist_out, dev_status, w
     return lib().varrate_anchor_search(ctypes.byref(cfg), _ptr(k), _ptr(v), stride, c, _ptr(idx_out),
                                        _ptr(dist_out), _ptr(dev_status), _ptr(ws), _nbytes(ws),
                                        _stream(stream))
+
+
+def varrate_anchor_residual(cfg, k, v, stride, c, idx, e_out, dev_status, stream=None) -> int:
+    return lib().varrate_anchor_residual(ctypes.byref(cfg), _ptr(k), _ptr(v), stride, c, _ptr(idx),
+                                         _ptr(e_out), _ptr(dev_status), _stream(stream))
 
 
 def varrate_decode_window(cfg, packed, basis_k, basis_v, q, n_q, layer, tail_k, tail_v, n_tail, out,

@@ -253,3 +253,22 @@ def test_anchor_search_host_checks(vlib):
     assert call(ws=None) == vlib.ERR_WORKSPACE
     f32 = vlib.make_config(2, 8, 4, 1000, batch=3, dtype=vlib.F32)
     assert call(c=f32) == vlib.ERR_UNSUPPORTED
+
+
+def test_anchor_residual_host_checks(vlib):
+    """Argument checks of the residual entry point, made before any launch."""
+    L = vlib.lib()
+    cfg = vlib.make_config(2, 8, 4, 1000, batch=3, dtype=vlib.BF16)
+
+    def call(c=cfg, k=A, v=A, stride=16, n=4, idx=A, e=A):
+        return L.varrate_anchor_residual(vlib.ctypes.byref(c), k, v, stride, n, idx, e, None, None)
+    assert call(k=None) == vlib.ERR_ARG
+    assert call(idx=None) == vlib.ERR_ARG
+    assert call(e=None) == vlib.ERR_ARG
+    assert call(stride=0) == vlib.ERR_ARG
+    assert call(stride=1001) == vlib.ERR_ARG
+    assert call(n=0) == vlib.ERR_ARG
+    assert call(n=9) == vlib.ERR_UNSUPPORTED
+    assert call(e=A + 2) == vlib.ERR_ARG
+    f32 = vlib.make_config(2, 8, 4, 1000, batch=3, dtype=vlib.F32)
+    assert call(c=f32) == vlib.ERR_UNSUPPORTED

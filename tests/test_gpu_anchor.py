@@ -122,3 +122,59 @@ def test_anchor_search_full_size_llama_layer():
     anchors = rows[rows % stride == 0]
     assert (idx[0, 0, anchors, 0] == anchors // stride).all()
     print(f"full size: worst distance error {worst:.3g} of the bar")
+
+
+def _residual(wl, k, v, stride, c, idx_dev):
+    cfg = V.make_config(wl.n_layers, wl.n_kv_heads, wl.group, wl.n_ctx, batch=wl.batch,
+                        window=min(wl.window, wl.n_ctx), dtype=V.BF16)
+    D = 2 * wl.n_kv_heads * wl.head_dim
+    e = torch.full((wl.batch, wl.n_layers, wl.n_ctx, D), float("nan"), dtype=torch.bfloat16, device="cuda")
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    V.check(V.varrate_anchor_residual(cfg, k, v, stride, c, idx_dev, e, status), "varrate_anchor_residual")
+    torch.cuda.synchronize()
+    return e, int(status.item())
+
+
+@pytest.mark.parametrize("name", ["llama_g2", "qwen_g4_s7", "few_anchors"])
+def test_anchor_residual_matches_oracle(name):
+    """Eq. 2 on the GPU's own anchor lists: e_t = z_t - mean of the listed anchors, against the
+    oracle's residual in fp64. Bar per coordinate: twice the bf16 rounding of the result (unit
+    roundoff 2^-8, so 2^-7 |want|) plus the fp32 rounding of the sum (2^-20 (|z_t| + the listed
+    anchors' magnitudes)). A numpy emulation of the kernel's arithmetic reaches 0.50 of this bar;
+    a dropped anchor mean or a wrong divisor exceed it by four orders of magnitude."""
+    wl, stride, c = CASES[name]
+    k, v, _, _, _ = synth.stack_inputs(wl, device="cuda")
+    idx, _ = _search(wl, k, v, stride, c)
+    e, st = _residual(wl, k, v, stride, c, torch.as_tensor(idx, device="cuda"))
+    assert st == 0, V.status_string(st)
+    got = e.to(torch.float64).cpu().numpy()
+    kc, vc = k.cpu(), v.cpu()
+    for b in range(wl.batch):
+        for l in range(wl.n_layers):
+            z = J.joint_vector(kc[b, l].double().numpy(), vc[b, l].double().numpy())
+            lists = idx[b, l].astype(np.int64)
+            want = J.residual(z, lists, stride)
+            mag = np.abs(z).copy()
+            for s in range(c):
+                ok = lists[:, s] >= 0
+                mag[ok] += np.abs(z[lists[ok, s] * stride])
+            bar = 2.0 ** -7 * np.abs(want) + 2.0 ** -20 * mag
+            err = np.abs(got[b, l] - want)
+            assert (err <= bar).all(), (name, b, l, float((err / np.maximum(bar, 1e-30)).max()))
+
+
+def test_anchor_residual_rejects_a_bad_list():
+    """An anchor number past the anchor count is caught by the kernel's own check: the call raises
+    VARRATE_ERR_CORRUPT, leaves that token's row unwritten and writes the others."""
+    wl, stride, c = CASES["llama_g2"]
+    k, v, _, _, _ = synth.stack_inputs(wl, device="cuda")
+    idx, _ = _search(wl, k, v, stride, c)
+    n_a = J.anchor_positions(wl.n_ctx, stride).size
+    bad = idx.copy()
+    bad[0, 0, 5, 1] = n_a + 3
+    e, st = _residual(wl, k, v, stride, c, torch.as_tensor(bad, device="cuda"))
+    assert st == V.ERR_CORRUPT
+    assert torch.isnan(e[0, 0, 5].float()).all()
+    good, st2 = _residual(wl, k, v, stride, c, torch.as_tensor(idx, device="cuda"))
+    assert st2 == 0
+    np.testing.assert_array_equal(e[0, 0, 6].float().cpu().numpy(), good[0, 0, 6].float().cpu().numpy())
