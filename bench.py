@@ -645,26 +645,34 @@ def sweep_anchor_search(V, wl, dev, stream, stride=16, c=4):
 
 
 def run_sweep(args, peak):
-    """The other seeded configurations, each with its own encode and decode numbers."""
+    """The other seeded configurations, each with its own encode and decode numbers. A configuration
+    that raises is reported under its key as {"error": ...}; the headline line is printed anyway."""
     from paper_2607_15498_gb300 import varrate as V
     dev = torch.device("cuda", torch.cuda.current_device())
     stream = torch.cuda.current_stream()
     out = {}
-    wl = synth.workload("llama1")
+
+    def run(key, fn):
+        try:
+            out[key] = fn()
+        except Exception as e:  # noqa: BLE001 - recorded in the JSON line, not hidden
+            out[key] = {"error": f"{type(e).__name__}: {e}"}
+            torch.cuda.empty_cache()
+
     per_call = 27.4e6
     copies = int(np.ceil(3 * l2_bytes(dev) / per_call))
-    out["llama1"] = sweep_config(V, wl, dev, peak, stream, decode_steps=256, copies=copies,
-                                 flush=True, enc_reps=5)
+    run("llama1", lambda: sweep_config(V, synth.workload("llama1"), dev, peak, stream, decode_steps=256,
+                                       copies=copies, flush=True, enc_reps=5))
     for kappa in synth.workload("qwen").budgets:
-        out[f"qwen_kappa{kappa:.2f}"] = sweep_config(V, synth.workload("qwen", budget_frac=kappa),
-                                                     dev, peak, stream, decode_steps=32)
+        run(f"qwen_kappa{kappa:.2f}", lambda kappa=kappa: sweep_config(
+            V, synth.workload("qwen", budget_frac=kappa), dev, peak, stream, decode_steps=32))
     wl = synth.workload("reuse")
-    out["reuse"] = sweep_reuse(V, wl, dev, peak, stream, n_batches=args.reuse_batches,
-                               n_window=32, n_decode=wl.decode_steps)
-    out["llama32_quantized"] = sweep_quant(V, synth.workload("llama32", n_layers=4), dev, peak,
-                                           stream, decode_steps=32)
-    out["joint_anchor_search"] = sweep_anchor_search(V, synth.workload("llama32", n_layers=4, batch=2),
-                                                     dev, stream)
+    run("reuse", lambda: sweep_reuse(V, wl, dev, peak, stream, n_batches=args.reuse_batches,
+                                     n_window=32, n_decode=wl.decode_steps))
+    run("llama32_quantized", lambda: sweep_quant(V, synth.workload("llama32", n_layers=4), dev, peak,
+                                                 stream, decode_steps=32))
+    run("joint_anchor_search", lambda: sweep_anchor_search(
+        V, synth.workload("llama32", n_layers=4, batch=2), dev, stream))
     return out
 
 
