@@ -644,6 +644,47 @@ def sweep_anchor_search(V, wl, dev, stream, stride=16, c=4):
     return res
 
 
+def sweep_anchor_residual(V, wl, dev, peak, stream, stride=16, c=4):
+    """Joint codec: the residuals e_t = z_t - mean of the token's nearest anchors (Sec. 3.1, Eq. 2)
+    over every (sequence, layer) of a Llama-shaped stack, on the lists of the search. Algorithmic
+    bytes per (sequence, layer): K and V read once (2 G N d bf16), the lists (N c int32) and the
+    residuals written (N 2 G d bf16); the anchors' rows come from L2 and are not counted."""
+    cfg = V.make_config(wl.n_layers, wl.n_kv_heads, wl.group, wl.n_ctx, batch=wl.batch,
+                        window=wl.window, dtype=V.BF16)
+    k, v, _, _, _ = synth.stack_inputs(wl, device=dev)
+    B, L, N, G, d = wl.batch, wl.n_layers, wl.n_ctx, wl.n_kv_heads, wl.head_dim
+    idx = torch.empty((B, L, N, c), dtype=torch.int32, device=dev)
+    dist = torch.empty((B, L, N, c), dtype=torch.float32, device=dev)
+    ws = torch.zeros(V.varrate_anchor_search_ws_bytes(cfg, stride), dtype=torch.uint8, device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    V.check(V.varrate_anchor_search(cfg, k, v, stride, c, idx, dist, status, ws, stream),
+            "varrate_anchor_search")
+    del dist, ws
+    e = torch.empty((B, L, N, 2 * G * d), dtype=torch.bfloat16, device=dev)
+    times = []
+    for i in range(6):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        V.check(V.varrate_anchor_residual(cfg, k, v, stride, c, idx, e, status, stream),
+                "varrate_anchor_residual")
+        e1.record(stream)
+        torch.cuda.synchronize()
+        if i >= 2:
+            times.append(e0.elapsed_time(e1))
+    ms = statistics.median(times)
+    units = B * L
+    nbytes = units * (2 * G * N * d * 2 + N * c * 4 + N * 2 * G * d * 2)
+    gbs = nbytes / (ms * 1e-3) / 1e9
+    res = {"workload": workload_desc(wl), "stride": stride, "c": c, "ms_per_layer": round(ms / units, 4),
+           "bytes_per_layer": int(nbytes // units), "gbs": round(gbs, 1),
+           "frac_of_hbm_peak": round(gbs / peak, 4), "status": V.status_string(int(status.item())),
+           "kernels": "one residual kernel per call (a warp per token), on the lists of one search call "
+                      "made before the timed calls"}
+    del k, v, idx, e
+    torch.cuda.empty_cache()
+    return res
+
+
 def run_sweep(args, peak):
     """The other seeded configurations, each with its own encode and decode numbers. A configuration
     that raises is reported under its key as {"error": ...}; the headline line is printed anyway."""
@@ -673,6 +714,8 @@ def run_sweep(args, peak):
                                                  stream, decode_steps=32))
     run("joint_anchor_search", lambda: sweep_anchor_search(
         V, synth.workload("llama32", n_layers=4, batch=2), dev, stream))
+    run("joint_anchor_residual", lambda: sweep_anchor_residual(
+        V, synth.workload("llama32", n_layers=4, batch=2), dev, peak, stream))
     return out
 
 
