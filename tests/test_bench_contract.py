@@ -23,3 +23,38 @@ def test_reference_arm_prints_one_contract_line():
     cb = d["cpu_baseline"]
     assert cb["kind"] == "oracle" and cb["value"] == d["value"] and cb["cores"] >= 1 and cb["sample"]
     assert "workload" in d["config"]
+
+
+def test_sweep_reports_a_failing_configuration_and_carries_on(monkeypatch):
+    """run_sweep on CPU with every configuration replaced by a stub: a configuration that raises is
+    reported under its own key as an error, and every later configuration still runs."""
+    import types
+
+    import torch
+
+    sys.path.insert(0, ROOT)
+    import bench
+    monkeypatch.setattr(torch.cuda, "current_device", lambda: 0)
+    monkeypatch.setattr(torch.cuda, "current_stream", lambda: None)
+    monkeypatch.setattr(torch.cuda, "empty_cache", lambda: None)
+    monkeypatch.setattr(bench, "l2_bytes", lambda dev: 129 << 20)
+    ran = []
+
+    def stub(name, fail=False):
+        def f(*a, **k):
+            ran.append(name)
+            if fail:
+                raise RuntimeError("planted")
+            return {"ok": name}
+        return f
+    monkeypatch.setattr(bench, "sweep_config", stub("config"))
+    monkeypatch.setattr(bench, "sweep_reuse", stub("reuse", fail=True))
+    monkeypatch.setattr(bench, "sweep_quant", stub("quant"))
+    monkeypatch.setattr(bench, "sweep_anchor_search", stub("anchor_search"))
+    monkeypatch.setattr(bench, "sweep_anchor_residual", stub("anchor_residual"))
+    out = bench.run_sweep(types.SimpleNamespace(reuse_batches=16), 6686.8)
+    assert out["reuse"] == {"error": "RuntimeError: planted"}
+    assert ran == ["config"] * 5 + ["reuse", "quant", "anchor_search", "anchor_residual"]
+    assert set(out) == {"llama1", "qwen_kappa0.10", "qwen_kappa0.20", "qwen_kappa0.30",
+                        "qwen_kappa0.50", "reuse", "llama32_quantized", "joint_anchor_search",
+                        "joint_anchor_residual"}
