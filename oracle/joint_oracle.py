@@ -141,6 +141,22 @@ def joint_ranks(sal32: np.ndarray, n_ctx: int, dim: int, rank_cap: int, stride: 
     return ranks, status, total, bc
 
 
+def joint_footprint(n_ctx: int, dim: int, stride: int, window: int, budget_frac: float, c: int,
+                    coef_bits: float = 16.0, group: int = 32, param_bits: int = 32,
+                    index_bytes: int = 2, elem_bytes: int = 2) -> float:
+    """Stored bytes of one (sequence, layer) under the joint codec as a fraction of the full cache
+    (N D values of elem_bytes): the exact set whole (|E| D values), the coded budget B of Eq. 3 in
+    coefficients of coef_bits bits (quantized: plus param_bits of group parameters per group of
+    ``group`` coefficients; coef_bits = 16 means unquantized), and c anchor indices of index_bytes
+    per coded token (Sec. 3.1, Budget: the indices are counted in the reported footprint)."""
+    exact = int(exact_mask(n_ctx, stride, window).sum())
+    coded = n_ctx - exact
+    b = joint_budget(n_ctx, dim, exact, budget_frac)
+    per_coef = coef_bits / 8.0 if coef_bits >= 16 else (coef_bits + param_bits / group) / 8.0
+    total = exact * dim * elem_bytes + max(b, 0) * per_coef + coded * c * index_bytes
+    return total / (n_ctx * dim * elem_bytes)
+
+
 # ------------------------------------------------ projection and reconstruction (Eq. 5)
 
 def joint_project(e: np.ndarray, basis: np.ndarray) -> np.ndarray:

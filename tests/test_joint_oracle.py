@@ -295,3 +295,18 @@ def test_encode_joint_at_kappa_one_reconstructs_exactly():
     assert (enc["ranks"][~exact] == D).all() and (enc["ranks"][exact] == 0).all()
     zh = J.joint_reconstruct(enc["z"], enc["idx"], enc["coef"], enc["ranks"], V, 8)
     np.testing.assert_allclose(zh, J.joint_vector(k, v), atol=1e-12)
+
+
+def test_footprint_matches_the_papers_measured_memory():
+    # Table "Coefficient quantization sweep" (Llama, keep 20 %): memory ~20 % in fp16, ~14 % with
+    # 8-bit, ~10 % with 4-bit and ~9 % with 3-bit coefficients; Sec. 3.1 "Budget": the anchor
+    # indices add 0.2 % of the cache. Paper setting: D = 2 x 8 x 128, stride 16, c = 4, w = 64; a
+    # 16K context; group parameters of two fp16 values per 32 coefficients.
+    n, D, stride, w, kappa, c = 16384, 2048, 16, 64, 0.2, 4
+    for bits, paper in ((16, 20.0), (8, 14.0), (4, 10.0), (3, 9.0)):
+        got = 100 * J.joint_footprint(n, D, stride, w, kappa, c, coef_bits=bits)
+        assert abs(got - paper) <= 1.5, (bits, got)
+    idx = 100 * (J.joint_footprint(n, D, stride, w, kappa, c) - J.joint_footprint(n, D, stride, w, kappa, 0))
+    assert 0.15 <= idx <= 0.25
+    # the budget is matched: without quantization or indices the footprint is kappa up to the floor
+    assert abs(J.joint_footprint(n, D, stride, w, kappa, 0) - kappa) < 1e-6
